@@ -1,0 +1,413 @@
+#!/usr/bin/env python3
+"""Decode-step benchmark of refusal-gated decoding on GB300.
+
+One step = one pass of the whole hot path over one batch of the Llama-3-8B-shaped
+workload (16 prompts x (1 greedy probe + 4 high-temperature sample rows), prompts
+U[512, 2048] tokens, suffixes U[0, 256], 32 q / 8 kv heads, head dim 128, bf16 KV
+in 16-token pages, fp32 logits over 128256): shared-prefix split-KV attention,
+the sample head (argmax / temperature + min-p + Philox draw) and the trie gate.
+Inputs are seeded synthetic data resident in HBM; L2 is flushed (256 MiB write)
+before every timed step, outside the timed events.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle on the
+host cores on a bounded sample of the same workload.  Under torchrun (N > 1)
+every rank runs its own batch (weak scaling, no collective in the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+os.environ.setdefault("OMP_NUM_THREADS", "1")
+os.environ.setdefault("OPENBLAS_NUM_THREADS", "1")
+os.environ.setdefault("MKL_NUM_THREADS", "1")
+
+import numpy as np  # noqa: E402
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode-step rows/sec and achieved HBM GB/s (% of GB300 peak), 1 GPU"
+UNIT = "rows/s"
+WORKLOAD = ("llama8b-shaped decode step: 16 prompts x (1 probe + 4 sample rows), prompt len U[512,2048], "
+            "suffix len U[0,256], 32 q / 8 kv heads, head dim 128, bf16 KV in 16-token pages, "
+            "fp32 Zipf(1.1) logits over 128256, T in {1,1.5,2,3}, min-p in {0.05,0.1}, 64 refusal seqs")
+FALLBACK_HBM_GBS = 6800.0
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def algorithmic_bytes(case):
+    """Bytes the method must read per step: prompt KV once per active group (all kv
+    heads), suffix KV once per active row, logits once per active row."""
+    a, h = case.attn, case.head
+    kv_tok = a.num_kv_heads * 2 * a.head_dim * 2
+    rpg = a.rows_per_group
+    attn = 0
+    for g in range(a.num_groups):
+        if a.row_active[g * rpg:(g + 1) * rpg].any():
+            attn += int(a.prompt_len[g]) * kv_tok
+    attn += int(sum(int(a.suffix_len[r]) * kv_tok for r in range(a.num_rows) if a.row_active[r]))
+    es = 4 if h.dtype == "f32" else 2
+    head = int(h.row_active.sum()) * h.vocab * es
+    return attn, head
+
+
+def _kernel_hash():
+    src = os.path.join(ROOT, "paper_2607_20791_gb300", "csrc", "attention.cu")
+    return hashlib.sha256(open(src, "rb").read()).hexdigest()[:12]
+
+
+def _profiled_traffic():
+    """Per-launch DRAM bytes of the attention kernel from the committed ncu summary,
+    if it was taken on the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", "attn_split_kernel_llama8b.md")
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    m = re.search(r"traffic_bytes_per_launch:\s*([0-9]+)\s*\(attention\.cu sha256 ([0-9a-f]+)\)", text)
+    if not m or m.group(2) != _kernel_hash():
+        return None
+    return int(m.group(1))
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples while the timed region runs."""
+
+    FIELDS = ("index,timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.25)
+        return self
+
+    def __exit__(self, *exc):
+        time.sleep(0.25)
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        try:
+            for line in open(self.path):
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 10:
+                    rows.append(parts)
+        except OSError:
+            pass
+        finally:
+            try:
+                os.unlink(self.path)
+            except OSError:
+                pass
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"], "samples": 0}
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+
+        sm = [num(r[2]) for r in rows if num(r[2]) is not None]
+        smax = [num(r[3]) for r in rows if num(r[3]) is not None]
+        reasons = set()
+        for r in rows:
+            for name, col in (("hw_slowdown", 6), ("hw_thermal_slowdown", 7), ("sw_thermal_slowdown", 8),
+                              ("sw_power_cap", 9)):
+                if r[col].lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(rows)}
+
+
+def _dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (cpu_baseline leg and --impl reference)
+# ---------------------------------------------------------------------------
+def _oracle_step(case, groups):
+    from oracle import attention as oattn
+    from oracle import gate as ogate
+    from oracle import sampling as osamp
+    rpg = case.attn.rows_per_group
+    rows = [g * rpg + i for g in groups for i in range(rpg)]
+    oattn.decode_attention_case(case.attn, rows=rows)
+    res = osamp.sample_head(case.head.logits, case.head.dtype, case.head.is_probe, case.head.temperature,
+                            case.head.min_p, case.head.seed, case.head.step, case.head.row_active, rows=rows)
+    probe = np.array([[res.tokens[g * rpg]] for g in groups], np.int32)
+    ogate.run_gate(probe, case.gate.refusal_seqs, case.gate.eos, case.gate.max_len)
+    return len(rows)
+
+
+def cpu_baseline(case, budget_s: float = 12.0):
+    """The oracle as it stands, single-threaded, on whole prompt groups of the step
+    until about `budget_s` seconds of CPU work; rows/s scaled from that sample."""
+    t0 = time.perf_counter()
+    rows = 0
+    g = 0
+    while time.perf_counter() - t0 < budget_s and g < case.attn.num_groups:
+        rows += _oracle_step(case, [g])
+        g += 1
+    dt = time.perf_counter() - t0
+    return {"value": rows / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{g} of {case.attn.num_groups} prompt groups ({rows} rows) of one step, fp64 NumPy, "
+                      f"{dt:.1f} s"}
+
+
+def run_reference(args):
+    world, rank, _ = _dist_env()
+    if rank != 0:
+        return
+    from paper_2607_20791_gb300 import workloads
+    case = workloads.llama8b(seed=0)
+    G = case.attn.num_groups
+    for i in range(args.warmup):
+        _oracle_step(case, [i % G])
+    times, rows = [], 0
+    for i in range(args.steps):
+        t0 = time.perf_counter()
+        rows += _oracle_step(case, [i % G])
+        times.append(time.perf_counter() - t0)
+    total = sum(times)
+    value = rows / total
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * total / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": WORKLOAD, "sample": "one prompt group (5 rows) of the step per timed step"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": "one prompt group (5 rows) per step, fp64 NumPy oracle, single thread"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+def run_ours(args):
+    import torch
+    world, rank, local = _dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_20791_gb300 import binding, device, workloads
+
+    case = workloads.llama8b(seed=rank)
+    attn_bytes, head_bytes = algorithmic_bytes(case)
+    step_bytes = attn_bytes + head_bytes
+    G, rpg = case.attn.num_groups, case.attn.rows_per_group
+    R = G * rpg
+    rows_per_step = int(case.head.row_active.sum())
+
+    att = device.attn_to_device(case.attn, device=dev)
+    head = device.head_to_device(case.head, device=dev)
+    trie = binding.Trie(case.gate.refusal_seqs, 2)
+    gstate = binding.new_gate_state(G, device=dev)
+    gate_active = torch.ones(R, dtype=torch.uint8, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def attn_call():
+        att.run(stream=stream.cuda_stream)
+
+    def head_gate_call():
+        binding.rgd_sample_head(head.logits, head.is_probe, head.temperature, head.min_p, head.seed, head.step,
+                                head.row_active, head.token_out, head.kept_count, None, head.dev_status,
+                                stream=stream.cuda_stream)
+        # the gate runs on the probe rows' tokens; its state is reset each step so
+        # every step gates the same first probe token (the step is timed alone)
+        binding.rgd_gate_state_init(gstate, G, stream=stream.cuda_stream)
+        binding.rgd_probe_gate(trie, G, rpg, head.token_out, 1, rpg, case.gate.eos, case.gate.max_len, gstate,
+                               gate_active, head.dev_status, stream=stream.cuda_stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(3):  # eager warm-up (also sets kernel attributes before capture)
+            attn_call()
+            head_gate_call()
+        torch.cuda.synchronize()
+        g_attn, g_hg = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_attn, stream=stream):
+            attn_call()
+        with torch.cuda.graph(g_hg, stream=stream):
+            head_gate_call()
+        torch.cuda.synchronize()
+    launches_per_step = 4  # attention, sample head, gate-state reset, gate
+
+    def one_step(ev):
+        flush.fill_(1)
+        ev[0].record(stream)
+        g_attn.replay()
+        ev[1].record(stream)
+        g_hg.replay()
+        ev[2].record(stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            one_step([torch.cuda.Event(enable_timing=True) for _ in range(3)])
+        torch.cuda.synchronize()
+
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        with torch.cuda.stream(stream):
+            for i in range(args.steps):
+                one_step(events[i])
+        torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    step_ms = [ev[0].elapsed_time(ev[2]) for ev in events]
+    attn_ms = [ev[0].elapsed_time(ev[1]) for ev in events]
+    hg_ms = [ev[1].elapsed_time(ev[2]) for ev in events]
+    mean_step = sum(step_ms) / len(step_ms)
+    mean_attn = sum(attn_ms) / len(attn_ms)
+    status = int(att.dev_status.item()) | int(head.dev_status.item())
+
+    # ---- end to end through the public API with host buffers ----------------
+    h2d_src = {
+        "q": case.attn.q, "logits": case.head.logits, "prompt_block_table": case.attn.prompt_block_table,
+        "prompt_len": case.attn.prompt_len, "suffix_block_table": case.attn.suffix_block_table,
+        "suffix_len": case.attn.suffix_len, "row_active": case.attn.row_active,
+        "temperature": case.head.temperature, "min_p": case.head.min_p, "seed": case.head.seed.view(np.int64),
+        "is_probe": case.head.is_probe}
+    dst = {"q": att.q, "logits": head.logits, "prompt_block_table": att.prompt_block_table,
+           "prompt_len": att.prompt_len, "suffix_block_table": att.suffix_block_table,
+           "suffix_len": att.suffix_len, "row_active": att.row_active, "temperature": head.temperature,
+           "min_p": head.min_p, "seed": head.seed, "is_probe": head.is_probe}
+    pinned = {}
+    for k, a in h2d_src.items():
+        t = torch.from_numpy(np.ascontiguousarray(a))
+        if dst[k].dtype != t.dtype:
+            t = t.view(dst[k].dtype)
+        pinned[k] = t.reshape(dst[k].shape).pin_memory()
+    h2d_bytes = sum(t.numel() * t.element_size() for t in pinned.values())
+    tok_host = torch.empty(R, dtype=torch.int32).pin_memory()
+    st_host = torch.empty_like(gstate, device="cpu").pin_memory()
+    d2h_bytes = tok_host.numel() * 4 + st_host.numel()
+    e2e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(args.steps)]
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup + args.steps):
+            flush.fill_(1)
+            if i >= args.warmup:
+                e2e_ev[i - args.warmup][0].record(stream)
+            for k, t in pinned.items():
+                dst[k].copy_(t, non_blocking=True)
+            g_attn.replay()
+            g_hg.replay()
+            tok_host.copy_(head.token_out, non_blocking=True)
+            st_host.copy_(gstate, non_blocking=True)
+            if i >= args.warmup:
+                e2e_ev[i - args.warmup][1].record(stream)
+        torch.cuda.synchronize()
+    e2e_ms = sum(a.elapsed_time(b) for a, b in e2e_ev) / args.steps
+
+    # ---- max over ranks --------------------------------------------------------
+    vals = torch.tensor([mean_step, e2e_ms, mean_attn], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(vals, op=dist.ReduceOp.MAX)
+    mean_step, e2e_ms, mean_attn = [float(x) for x in vals.tolist()]
+    value = world * rows_per_step / (mean_step / 1e3)
+    e2e_value = world * rows_per_step / (e2e_ms / 1e3)
+
+    if rank == 0:
+        peak, peak_kind = _peaks()
+        attn_gbs = attn_bytes / (mean_attn / 1e3) / 1e9
+        step_gbs = step_bytes / (mean_step / 1e3) / 1e9
+        traffic = _profiled_traffic()
+        cpu = cpu_baseline(case) if world == 1 else None
+        clocks = clk.summary()
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": mean_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "rows_per_step": rows_per_step, "groups": G,
+                       "l2": "flushed between steps (256 MiB write, outside the timed events)",
+                       "timing": "CUDA events per step on the launching stream; step = attention graph + "
+                                 "sample-head/gate graph", "parallelism": f"replicas x{world}"},
+            "step_hbm_gbs": step_gbs, "step_hbm_frac": step_gbs / peak,
+            "step_algorithmic_bytes": step_bytes,
+            "kernels_ms": {"attention": mean_attn, "sample_head_and_gate": sum(hg_ms) / len(hg_ms)},
+            "roofline": {"bound": "hbm", "kernel": "attn_split_kernel<128>", "achieved": attn_gbs,
+                         "peak": peak, "unit": "GB/s", "frac": attn_gbs / peak, "traffic": traffic,
+                         "algorithmic_bytes": attn_bytes, "peak_source": peak_kind},
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
+                    "d2h_bytes_per_step": d2h_bytes, "ms_per_step": e2e_ms},
+            "gpu_launches": launches_per_step * args.steps,
+            "clocks": clocks, "dev_status": status,
+        }
+        print(json.dumps(line), flush=True)
+    trie.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    args = ap.parse_args()
+    args.warmup = max(3, args.warmup)
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

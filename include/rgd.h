@@ -1,0 +1,220 @@
+/*
+ * rgd.h -- C ABI of the refusal-gated decode step on GB300 (sm_103a).
+ *
+ * Refusal-gated decoding (arxiv 2607.20791) runs, for every prompt, one greedy
+ * "probe" row and N high-temperature sample rows.  All rows of a prompt attend
+ * to the prompt's KV cache, which is computed once and reused (Sec. 3), plus
+ * their own generated-suffix KV.  The greedy probe is checked token by token
+ * against a set P of refusal prefixes (the compatibility predicate C, Sec. 3;
+ * token-prefix matching with a two-token minimum, App. D); the hard gate of
+ * Alg. 1 then either keeps the greedy refusal or discards the probe and keeps
+ * the high-temperature samples.
+ *
+ * This library implements one decode step of that loop as CUDA kernels:
+ *   rgd_prefix_decode_attn  shared-prefix split-KV decode attention,
+ *   rgd_sample_head         greedy argmax / temperature + min-p + Philox sample,
+ *   rgd_probe_gate          per-token refusal-prefix gate on a token trie.
+ *
+ * Conventions for every entry point
+ *   - Tensor pointers are DEVICE pointers owned by the caller unless a comment
+ *     says "host".  The library never frees them.  bf16 values are passed as
+ *     their 16-bit patterns (rgd_bf16).  All tensors are dense, row-major, with
+ *     the shapes given, and 16-byte aligned base addresses.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = the legacy
+ *     default stream) and use the device that is current on the calling thread.
+ *   - The return value is a host status: RGD_OK, or an RGD_ERR_* code when the
+ *     arguments are rejected (nothing is launched) or a launch fails;
+ *     rgd_last_error_string() then describes the error (per thread).
+ *   - Errors found on the device (an out-of-range page id, an invalid
+ *     temperature, a wait that timed out) never trap: the kernel ORs an
+ *     RGD_DEV_* bit into *dev_status (a caller-owned device int32, may be NULL)
+ *     and skips the offending work.  Read it after synchronising.
+ */
+#ifndef RGD_H
+#define RGD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* host status codes */
+#define RGD_OK 0
+#define RGD_ERR_INVALID_ARG 1
+#define RGD_ERR_CUDA 2
+#define RGD_ERR_UNSUPPORTED 3
+
+/* device status bits (ORed into *dev_status) */
+#define RGD_DEV_BAD_PAGE 1      /* block-table entry outside [0, num_pages): read as zeros */
+#define RGD_DEV_BAD_TOKEN 2     /* negative probe token that is not the stop token: skipped */
+#define RGD_DEV_WAIT_TIMEOUT 4  /* a bounded wait on a copy gave up; outputs of that block are missing */
+#define RGD_DEV_BAD_PARAM 8     /* temperature < 0 or not finite, min_p outside [0, 1], or non-finite logits max */
+
+/* logits element types */
+#define RGD_F32 0
+#define RGD_BF16 1
+
+/* gate decisions (Sec. 3 / Alg. 1 outcomes) */
+#define RGD_PENDING 0
+#define RGD_REFUSAL 1      /* the greedy probe stays refusal-compatible: return the greedy refusal */
+#define RGD_NON_REFUSAL 2  /* the probe became incompatible: discard it, keep the samples */
+
+typedef uint16_t rgd_bf16;
+typedef void* rgd_stream_t;
+
+/* Description of the last error on this thread ("" if none). */
+const char* rgd_last_error_string(void);
+/* Library version string. */
+const char* rgd_version(void);
+
+/* ------------------------------------------------------------------------ */
+/* Shared-prefix decode attention (Sec. 3: prompt KV reused by the probe and   */
+/* the sampling stage; here read once per prompt group and kv head)            */
+/* ------------------------------------------------------------------------ */
+
+/* Shape of one attention call.  R = num_groups * rows_per_group rows; row
+ * g*rows_per_group is the probe of group g, the next rows_per_group-1 rows are
+ * its sample rows.  Query head j uses kv head j / (num_q_heads/num_kv_heads). */
+typedef struct {
+  int32_t num_groups;        /* G >= 1                                          */
+  int32_t rows_per_group;    /* 1 + N >= 1                                      */
+  int32_t num_q_heads;       /* Hq, a multiple of num_kv_heads                  */
+  int32_t num_kv_heads;      /* Hkv >= 1                                        */
+  int32_t head_dim;          /* D: 64 or 128                                    */
+  int32_t page_size;         /* tokens per KV page: 16                          */
+  int32_t num_pages;         /* pages in each of the K and V pools              */
+  int32_t max_prompt_pages;  /* columns of prompt_block_table (>= 1)            */
+  int32_t max_suffix_pages;  /* columns of suffix_block_table (>= 1)            */
+  int32_t prompt_splits;     /* KV splits per prompt; 0 = chosen by the library */
+  int32_t suffix_splits;     /* KV splits per suffix; 0 = chosen by the library */
+} rgd_attn_shape;
+
+/* Bytes of device workspace rgd_prefix_decode_attn needs for this shape. */
+size_t rgd_prefix_decode_attn_workspace_size(const rgd_attn_shape* shape);
+
+/* Decode attention of every active row over [prompt KV of its group | its own
+ * suffix KV] (the concatenation; no causal mask; no rotary embedding):
+ *   out[r, j, :] = softmax(softmax_scale * K q[r, j]) V,
+ *   lse[r, j]    = ln sum exp(softmax_scale * K q[r, j])   (natural log).
+ * Prompt KV of a group is split into prompt_splits ranges; each range is read
+ * once and attended by all (rows_per_group * Hq/Hkv) queries of that group and
+ * kv head; each row's suffix likewise in suffix_splits ranges; the partial
+ * results are merged by log-sum-exp.
+ *
+ *   q                  bf16 [R, Hq, D]
+ *   k_pages, v_pages   bf16 [num_pages, Hkv, page_size, D]
+ *   prompt_block_table int32 [G, max_prompt_pages]: page ids of prompt tokens
+ *                      (token t in page table[t / page_size], slot t % page_size)
+ *   prompt_len         int32 [G], 0 <= prompt_len <= max_prompt_pages*page_size
+ *   suffix_block_table int32 [R, max_suffix_pages]
+ *   suffix_len         int32 [R], 0 <= suffix_len <= max_suffix_pages*page_size
+ *   row_active         uint8 [R] or NULL (all active); inactive rows read no KV
+ *                      and their out/lse are left untouched
+ *   softmax_scale      > 0 (1/sqrt(D) for standard attention)
+ *   out                bf16 [R, Hq, D]; lse float [R, Hq] or NULL
+ *   workspace          device memory of rgd_prefix_decode_attn_workspace_size()
+ *                      bytes, 256-byte aligned, ZERO-FILLED before its first use;
+ *                      a successful call leaves it zero-filled again (re-zero it
+ *                      after a call that reported a device error).  Calls that
+ *                      share a workspace must not overlap in time.
+ * A group with prompt_len 0 and a row with suffix_len 0 are valid; a row with
+ * neither gets out = 0, lse = -inf.  Page ids outside [0, num_pages) read as
+ * zeros and set RGD_DEV_BAD_PAGE.  Lengths beyond the table are rejected on the
+ * device (RGD_DEV_BAD_PAGE) because the host does not read device lengths. */
+int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf16* q,
+                           const rgd_bf16* k_pages, const rgd_bf16* v_pages,
+                           const int32_t* prompt_block_table, const int32_t* prompt_len,
+                           const int32_t* suffix_block_table, const int32_t* suffix_len,
+                           const uint8_t* row_active, float softmax_scale, rgd_bf16* out,
+                           float* lse, void* workspace, size_t workspace_bytes,
+                           int32_t* dev_status, rgd_stream_t stream);
+
+/* ------------------------------------------------------------------------ */
+/* Sample head: G_M's greedy token and S_{T,theta}'s truncated sample          */
+/* (Sec. 3, Alg. 1; truncation = min-p, Sec. 1)                                */
+/* ------------------------------------------------------------------------ */
+
+/* For every active row r of logits [rows, vocab] (RGD_F32 or RGD_BF16):
+ *   greedy rows (is_probe[r] != 0 or temperature[r] == 0):
+ *     token = argmax, lowest index on ties; kept_count = 1.
+ *   sample rows: l_max = max logit; cutoff c = fl32(l_max + fl32(T ln p_min))
+ *     (T ln p_min evaluated in double, rounded once to float; p_min = 0 keeps
+ *     everything); kept set K = {i : l_i >= c} (this is {p_i >= p_min p_max}
+ *     for p = softmax(l/T)); w_i = exp((l_i - l_max)/T); u = Philox4x32-10
+ *     uniform with key = seed[r] (low word first) and counter = (step low,
+ *     step high, 0, 0): u = (word0 >> 8) * 2^-24; token = the smallest i in K
+ *     with sum_{j in K, j <= i} w_j > u * sum_K w.
+ *   token_out int32 [rows] (-1 for inactive rows and rejected parameters);
+ *   kept_count int32 [rows] or NULL: |K| (0 for inactive rows);
+ *   kept_mask uint8 [rows, vocab] or NULL: 1 where i in K (sample rows only;
+ *     rows that are greedy or inactive are not written).
+ * is_probe may be NULL (no probe rows); row_active may be NULL (all active).
+ * vocab must satisfy vocab * element size <= 8 * 200 KiB. */
+int rgd_sample_head(int32_t rows, int32_t vocab, int32_t dtype, const void* logits,
+                    const uint8_t* is_probe, const float* temperature, const float* min_p,
+                    const uint64_t* seed, uint64_t step, const uint8_t* row_active,
+                    int32_t* token_out, int32_t* kept_count, uint8_t* kept_mask,
+                    int32_t* dev_status, rgd_stream_t stream);
+
+/* ------------------------------------------------------------------------ */
+/* Refusal-prefix gate (compatibility predicate C, Sec. 3; hard gate, Alg. 1)  */
+/* ------------------------------------------------------------------------ */
+
+/* Token trie of the refusal-prefix set P, built on the host and uploaded to the
+ * current device.  Library-owned; release with rgd_trie_destroy. */
+typedef struct rgd_trie rgd_trie;
+
+/* tokens (host) int32 [offsets[n_seq]]: the sequences back to back, each token
+ * >= 0; offsets (host) int64 [n_seq + 1], offsets[0] = 0, strictly increasing
+ * (every sequence non-empty).  Duplicates and sequences that are prefixes of
+ * others are allowed.  min_confirm >= 1 is the minimum length of a refusal
+ * prefix whose full match confirms a refusal (2 in the paper, App. D).
+ * n_seq = 0 gives the empty set (every probe is incompatible). */
+int rgd_trie_create(const int32_t* tokens, const int64_t* offsets, int32_t n_seq,
+                    int32_t min_confirm, rgd_trie** out);
+int rgd_trie_destroy(rgd_trie* trie);
+/* Node and edge counts of a trie (root included). */
+int rgd_trie_info(const rgd_trie* trie, int32_t* num_nodes, int32_t* num_edges);
+
+/* Per-group gate state, in device memory owned by the caller. */
+typedef struct {
+  int32_t node;           /* trie node of the probe q (root = 0)                    */
+  int32_t length;         /* |q|: probe tokens appended (stop token excluded)        */
+  int32_t steps;          /* probe tokens consumed (stop token included)             */
+  int32_t decisive_step;  /* 0-based index of the token that decided; -1 if pending  */
+  uint8_t decision;       /* RGD_PENDING / RGD_REFUSAL / RGD_NON_REFUSAL             */
+  uint8_t confirmed;      /* some refusal prefix of length >= min_confirm prefixes q */
+  uint8_t done;           /* the probe has ended (stop token, length cap, discarded) */
+  uint8_t reserved;
+} rgd_gate_state;
+
+/* Reset `groups` states to the empty probe (node 0, pending). */
+int rgd_gate_state_init(rgd_gate_state* state, int32_t groups, rgd_stream_t stream);
+
+/* Feed n_tokens greedy probe tokens per group to the hard gate.  Token k of
+ * group g is probe_tokens[g * token_stride + k] (token_stride >= n_tokens; use
+ * the sample head's token_out with token_stride = rows_per_group and n_tokens =
+ * 1 to gate the probe row of every group).  For each token of a group whose
+ * probe has not ended:
+ *   - the stop token (eos_token >= 0) ends the probe: REFUSAL if q is
+ *     compatible (q non-empty, or P non-empty), else NON_REFUSAL;
+ *   - otherwise q <- q || y; if q is not compatible: NON_REFUSAL, the probe
+ *     ends; if a refusal prefix of length >= min_confirm is now a prefix of q:
+ *     confirmed, REFUSAL (the probe continues to produce its text); if |q|
+ *     reaches max_len: the probe ends, REFUSAL if still pending.
+ * Then row_active [groups*rows_per_group] (updated in place, may be NULL):
+ * the probe row is cleared once the probe has ended; the sample rows of a group
+ * are cleared once its decision is REFUSAL.  Negative tokens other than the
+ * stop token are skipped and set RGD_DEV_BAD_TOKEN. */
+int rgd_probe_gate(const rgd_trie* trie, int32_t groups, int32_t rows_per_group,
+                   const int32_t* probe_tokens, int32_t n_tokens, int64_t token_stride,
+                   int32_t eos_token, int32_t max_len, rgd_gate_state* state,
+                   uint8_t* row_active, int32_t* dev_status, rgd_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RGD_H */
