@@ -131,6 +131,31 @@ int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf16* q,
                            float* lse, void* workspace, size_t workspace_bytes,
                            int32_t* dev_status, rgd_stream_t stream);
 
+/* Allocation-free form of rgd_prefix_decode_attn (the paper has no counterpart;
+ * this is a deployment convenience).  Same arguments and results, minus the
+ * workspace: the split partials and merge tickets live in one fixed 8 MiB device
+ * array inside the library (one per device, held by every process that loads the
+ * library until it exits).  It is for callers that cannot call cudaMalloc: for
+ * example a serving engine whose KV-cache manager has already reserved the free
+ * device memory (a new allocation would fail or break its memory accounting),
+ * or a latency-critical decode loop where cudaMalloc / cudaFree would
+ * synchronise the device.  The caller still passes every input and output.
+ *   - Shapes whose workspace (rgd_prefix_decode_attn_workspace_size) exceeds
+ *     8 MiB are rejected with RGD_ERR_UNSUPPORTED.
+ *   - The first call on a device looks up the array's device address (once per
+ *     device, with that device current); make that first call before any stream
+ *     capture.
+ *   - Each call clears the tickets with cudaMemsetAsync on `stream`; nothing is
+ *     allocated.  Every call shares the one array and it keeps the last call's
+ *     contents, so calls that overlap on the GPU (other streams, other threads)
+ *     race: serialise them. */
+int rgd_prefix_decode_attn_noalloc(const rgd_attn_shape* shape, const rgd_bf16* q,
+                                   const rgd_bf16* k_pages, const rgd_bf16* v_pages,
+                                   const int32_t* prompt_block_table, const int32_t* prompt_len,
+                                   const int32_t* suffix_block_table, const int32_t* suffix_len,
+                                   const uint8_t* row_active, float softmax_scale, rgd_bf16* out,
+                                   float* lse, int32_t* dev_status, rgd_stream_t stream);
+
 /* ------------------------------------------------------------------------ */
 /* Sample head: G_M's greedy token and S_{T,theta}'s truncated sample          */
 /* (Sec. 3, Alg. 1; truncation = min-p, Sec. 1)                                */

@@ -54,6 +54,8 @@ _SIGNATURES = {
     "rgd_prefix_decode_attn_workspace_size": (_SZ, [ctypes.POINTER(AttnShape)]),
     "rgd_prefix_decode_attn": (ctypes.c_int, [ctypes.POINTER(AttnShape), _P, _P, _P, _P, _P, _P, _P, _P, _F,
                                                _P, _P, _P, _SZ, _P, _P]),
+    "rgd_prefix_decode_attn_noalloc": (ctypes.c_int, [ctypes.POINTER(AttnShape), _P, _P, _P, _P, _P, _P, _P,
+                                                       _P, _F, _P, _P, _P, _P]),
     "rgd_sample_head": (ctypes.c_int, [_I32, _I32, _I32, _P, _P, _P, _P, _P, _U64, _P, _P, _P, _P, _P, _P]),
     "rgd_trie_create": (ctypes.c_int, [_P, _P, _I32, _I32, ctypes.POINTER(_P)]),
     "rgd_trie_destroy": (ctypes.c_int, [_P]),
@@ -145,6 +147,22 @@ def rgd_prefix_decode_attn(shape: AttnShape, q, k_pages, v_pages, prompt_block_t
         _ptr(out, "out", torch.bfloat16), _ptr(lse, "lse", torch.float32, optional=True),
         _ptr(workspace, "workspace"), ws_bytes, _ptr(dev_status, "dev_status", torch.int32, optional=True),
         _stream(stream)))
+
+
+def rgd_prefix_decode_attn_noalloc(shape: AttnShape, q, k_pages, v_pages, prompt_block_table, prompt_len,
+                                   suffix_block_table, suffix_len, row_active, softmax_scale: float, out,
+                                   lse, dev_status=None, stream=None) -> None:
+    """Same as :func:`rgd_prefix_decode_attn` without a workspace: the library's
+    fixed device scratch is used (for callers that cannot allocate device memory)."""
+    import torch
+    _check(load_library().rgd_prefix_decode_attn_noalloc(
+        ctypes.byref(shape), _ptr(q, "q", torch.bfloat16), _ptr(k_pages, "k_pages", torch.bfloat16),
+        _ptr(v_pages, "v_pages", torch.bfloat16), _ptr(prompt_block_table, "prompt_block_table", torch.int32),
+        _ptr(prompt_len, "prompt_len", torch.int32),
+        _ptr(suffix_block_table, "suffix_block_table", torch.int32), _ptr(suffix_len, "suffix_len", torch.int32),
+        _ptr(row_active, "row_active", torch.uint8, optional=True), float(softmax_scale),
+        _ptr(out, "out", torch.bfloat16), _ptr(lse, "lse", torch.float32, optional=True),
+        _ptr(dev_status, "dev_status", torch.int32, optional=True), _stream(stream)))
 
 
 def rgd_sample_head(logits, is_probe, temperature, min_p, seed, step: int, row_active, token_out,

@@ -564,3 +564,61 @@ extern "C" int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf1
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? RGD_OK : cuda_error(e, "attention launch");
 }
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of rgd_prefix_decode_attn
+// ---------------------------------------------------------------------------
+// The split partials and tickets live in a fixed file-scope device array
+// instead of a caller-provided workspace.  The array exists once per device in
+// every process that loads the library, for the life of the process.
+namespace rgd {
+namespace {
+
+constexpr size_t kStaticScratchBytes = size_t(8) << 20;  // 8 MiB
+__device__ __align__(256) uint8_t g_attn_scratch[kStaticScratchBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+void* g_scratch_ptr[kMaxDevices] = {};
+
+}  // namespace
+}  // namespace rgd
+
+extern "C" int rgd_prefix_decode_attn_noalloc(const rgd_attn_shape* shape, const rgd_bf16* q,
+                                              const rgd_bf16* k_pages, const rgd_bf16* v_pages,
+                                              const int32_t* prompt_block_table, const int32_t* prompt_len,
+                                              const int32_t* suffix_block_table, const int32_t* suffix_len,
+                                              const uint8_t* row_active, float softmax_scale, rgd_bf16* out,
+                                              float* lse, int32_t* dev_status, rgd_stream_t stream) {
+  clear_error();
+  if (int rc = check_shape(shape)) return rc;
+  const WsLayout w = ws_layout(shape);
+  if (w.total > kStaticScratchBytes)
+    return set_error(RGD_ERR_UNSUPPORTED,
+                     "rgd_prefix_decode_attn_noalloc: this shape needs %zu bytes of scratch; the static "
+                     "scratch holds %zu (use rgd_prefix_decode_attn with a workspace)",
+                     w.total, kStaticScratchBytes);
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return set_error(RGD_ERR_UNSUPPORTED, "device ordinal %d >= %d", dev, kMaxDevices);
+  void* scratch = nullptr;
+  {
+    // once per device, with that device current: the host-side symbol is only a
+    // stand-in, so the kernel gets the device address of the array
+    std::lock_guard<std::mutex> lock(g_scratch_mu);
+    if (g_scratch_ptr[dev] == nullptr) {
+      void* p = nullptr;
+      e = cudaGetSymbolAddress(&p, g_attn_scratch);
+      if (e != cudaSuccess) return cuda_error(e, "cudaGetSymbolAddress(g_attn_scratch)");
+      g_scratch_ptr[dev] = p;
+    }
+    scratch = g_scratch_ptr[dev];
+  }
+  // the array keeps the previous call's contents: the tickets must start at zero
+  e = cudaMemsetAsync(scratch, 0, w.ml_off, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_error(e, "cudaMemsetAsync(scratch tickets)");
+  return rgd_prefix_decode_attn(shape, q, k_pages, v_pages, prompt_block_table, prompt_len, suffix_block_table,
+                                suffix_len, row_active, softmax_scale, out, lse, scratch, kStaticScratchBytes,
+                                dev_status, stream);
+}
