@@ -380,7 +380,7 @@ def run_ours(args):
             "step_hbm_gbs": step_gbs, "step_hbm_frac": step_gbs / peak,
             "step_algorithmic_bytes": step_bytes,
             "kernels_ms": {"attention": mean_attn, "sample_head_and_gate": sum(hg_ms) / len(hg_ms)},
-            "roofline": {"bound": "hbm", "kernel": "attn_split_kernel<128>", "achieved": attn_gbs,
+            "roofline": {"bound": "hbm", "kernel": "attn_persistent_kernel<128>", "achieved": attn_gbs,
                          "peak": peak, "unit": "GB/s", "frac": attn_gbs / peak, "traffic": traffic,
                          "algorithmic_bytes": attn_bytes, "peak_source": peak_kind},
             "cpu_baseline": cpu,

@@ -87,21 +87,23 @@ typedef struct {
   int32_t num_pages;         /* pages in each of the K and V pools              */
   int32_t max_prompt_pages;  /* columns of prompt_block_table (>= 1)            */
   int32_t max_suffix_pages;  /* columns of suffix_block_table (>= 1)            */
-  int32_t prompt_splits;     /* KV splits per prompt; 0 = chosen by the library */
-  int32_t suffix_splits;     /* KV splits per suffix; 0 = chosen by the library */
+  int32_t num_ctas;          /* persistent blocks; 0 = one per SM of the device  */
+  int32_t reserved;          /* must be 0                                       */
 } rgd_attn_shape;
 
-/* Bytes of device workspace rgd_prefix_decode_attn needs for this shape. */
+/* Bytes of device workspace rgd_prefix_decode_attn needs for this shape (it
+ * depends on the current device's SM count when num_ctas is 0). */
 size_t rgd_prefix_decode_attn_workspace_size(const rgd_attn_shape* shape);
 
 /* Decode attention of every active row over [prompt KV of its group | its own
  * suffix KV] (the concatenation; no causal mask; no rotary embedding):
  *   out[r, j, :] = softmax(softmax_scale * K q[r, j]) V,
  *   lse[r, j]    = ln sum exp(softmax_scale * K q[r, j])   (natural log).
- * Prompt KV of a group is split into prompt_splits ranges; each range is read
- * once and attended by all (rows_per_group * Hq/Hkv) queries of that group and
- * kv head; each row's suffix likewise in suffix_splits ranges; the partial
- * results are merged by log-sum-exp.
+ * Every prompt KV page of a group is read once and attended by all
+ * rows_per_group * Hq/Hkv queries of that group and kv head; a row's suffix
+ * pages are attended by that row's queries.  The pages of all (group, kv head)
+ * jobs are divided evenly over num_ctas persistent blocks; a job split across
+ * blocks is merged from its partial results by log-sum-exp.
  *
  *   q                  bf16 [R, Hq, D]
  *   k_pages, v_pages   bf16 [num_pages, Hkv, page_size, D]

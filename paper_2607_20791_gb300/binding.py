@@ -33,7 +33,7 @@ class RgdError(RuntimeError):
 class AttnShape(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "num_groups", "rows_per_group", "num_q_heads", "num_kv_heads", "head_dim", "page_size",
-        "num_pages", "max_prompt_pages", "max_suffix_pages", "prompt_splits", "suffix_splits")]
+        "num_pages", "max_prompt_pages", "max_suffix_pages", "num_ctas", "reserved")]
 
 
 class GateState(ctypes.Structure):

@@ -48,21 +48,21 @@ class DeviceAttn:
                                        self.dev_status, stream)
 
 
-def attn_shape(case: AttnCase, prompt_splits: int = 0, suffix_splits: int = 0) -> binding.AttnShape:
+def attn_shape(case: AttnCase, num_ctas: int = 0) -> binding.AttnShape:
     return binding.AttnShape(
         num_groups=case.num_groups, rows_per_group=case.rows_per_group,
         num_q_heads=case.num_q_heads, num_kv_heads=case.num_kv_heads, head_dim=case.head_dim,
         page_size=case.page_size, num_pages=case.num_pages,
         max_prompt_pages=case.prompt_block_table.shape[1],
         max_suffix_pages=case.suffix_block_table.shape[1],
-        prompt_splits=prompt_splits, suffix_splits=suffix_splits)
+        num_ctas=num_ctas, reserved=0)
 
 
-def attn_to_device(case: AttnCase, device="cuda", prompt_splits: int = 0, suffix_splits: int = 0,
+def attn_to_device(case: AttnCase, device="cuda", num_ctas: int = 0,
                    kv: Optional[tuple] = None) -> DeviceAttn:
     """Copy the case to `device`; `kv` may supply already-resident (k_pages, v_pages)."""
     import torch
-    shape = attn_shape(case, prompt_splits, suffix_splits)
+    shape = attn_shape(case, num_ctas)
     if kv is None:
         k = _t(case.k_pages, device, torch.bfloat16)
         v = _t(case.v_pages, device, torch.bfloat16)

@@ -38,6 +38,7 @@ def test_version_and_argument_errors_without_gpu(lib_path):
     assert lib.rgd_prefix_decode_attn_workspace_size(ctypes.byref(shape)) == 0
     assert b"head_dim" in lib.rgd_last_error_string()
     shape.head_dim = 128
+    shape.num_ctas = 8
     assert lib.rgd_prefix_decode_attn_workspace_size(ctypes.byref(shape)) > 0
     # null pointers are rejected on the host before any launch
     rc = lib.rgd_sample_head(4, 100, 0, None, None, None, None, None, 0, None, None, None, None, None, None)
@@ -46,11 +47,14 @@ def test_version_and_argument_errors_without_gpu(lib_path):
     assert rc == binding.RGD_ERR_INVALID_ARG
 
 
-def test_workspace_size_grows_with_splits(lib_path):
+def test_workspace_size_grows_with_blocks(lib_path):
     lib = binding.load_library(lib_path)
     s = binding.AttnShape(num_groups=16, rows_per_group=5, num_q_heads=32, num_kv_heads=8, head_dim=128,
-                          page_size=16, num_pages=2000, max_prompt_pages=128, max_suffix_pages=16)
+                          page_size=16, num_pages=2000, max_prompt_pages=128, max_suffix_pages=16, num_ctas=100)
     a = lib.rgd_prefix_decode_attn_workspace_size(ctypes.byref(s))
-    s.prompt_splits = 16
+    s.num_ctas = 400
     b = lib.rgd_prefix_decode_attn_workspace_size(ctypes.byref(s))
-    assert b > a > 0
+    # tickets for 128 jobs + (ctas + jobs - 1) partial slots of 20 queries x (128 + 2) floats
+    assert b - a == 300 * 20 * 128 * 4 + 300 * 20 * 8
+    s.reserved = 1
+    assert lib.rgd_prefix_decode_attn_workspace_size(ctypes.byref(s)) == 0

@@ -47,11 +47,13 @@ def _check(case, dev, rows=None, expect_status=0):
 
 
 @pytest.mark.parametrize("D", [64, 128])
-@pytest.mark.parametrize("splits", [(0, 0), (1, 1), (3, 2), (7, 5)])
-def test_small_multi_tile_ragged(gpu_lib, D, splits):
+@pytest.mark.parametrize("ctas", [0, 1, 2, 3, 7, 29, 64, 200])
+def test_small_multi_tile_ragged(gpu_lib, D, ctas):
+    # 1 block (every job in one block), a few blocks (jobs split at ragged page
+    # boundaries), and more blocks than pages (empty blocks, one-page pieces)
     case = workloads.make_attn_case("small", 3, 3, 8, 2, D, [0, 37, 300],
-                                    [0, 1, 16, 17, 40, 0, 5, 33, 64], seed=D + splits[0])
-    _check(case, _run(case, prompt_splits=splits[0], suffix_splits=splits[1]))
+                                    [0, 1, 16, 17, 40, 0, 5, 33, 64], seed=D + ctas)
+    _check(case, _run(case, num_ctas=ctas))
 
 
 def test_tiny_config(gpu_lib):
@@ -65,9 +67,10 @@ def test_llama8b_full(gpu_lib):
     _check(case, _run(case))
 
 
-def test_llama8b_many_splits(gpu_lib):
+@pytest.mark.parametrize("ctas", [13, 1000])
+def test_llama8b_other_block_counts(gpu_lib, ctas):
     case = workloads.llama8b(seed=1).attn
-    _check(case, _run(case, prompt_splits=17, suffix_splits=3), rows=list(range(0, 80, 7)))
+    _check(case, _run(case, num_ctas=ctas), rows=list(range(0, 80, 7)))
 
 
 def test_long_prompt_sampled_rows(gpu_lib):
@@ -86,7 +89,7 @@ def test_query_tiles_per_group(gpu_lib):
     for rpg, Hq in [(1, 32), (3, 64), (16, 64)]:
         case = workloads.make_attn_case("q", 2, rpg, Hq, 8, 128, [100, 260], list(range(0, 2 * rpg)),
                                         seed=rpg)
-        _check(case, _run(case, prompt_splits=2))
+        _check(case, _run(case, num_ctas=5))
 
 
 def test_masked_rows_and_groups(gpu_lib):

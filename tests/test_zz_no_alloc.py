@@ -48,8 +48,8 @@ def test_noalloc_matches_workspace_entry_point_twice(gpu_lib):
 
 def test_noalloc_rejects_oversized_shapes(gpu_lib):
     import torch
-    case = workloads.long_prompt(seed=0, with_kv=False).attn
-    shape = device.attn_shape(case)
+    case = workloads.high_batch(seed=0, with_kv=False).attn  # 2048 (group, kv head) jobs
+    shape = device.attn_shape(case, num_ctas=152)
     assert binding.rgd_prefix_decode_attn_workspace_size(shape) > (8 << 20)
     t = torch.zeros(16, dtype=torch.int32, device="cuda")
     b = torch.zeros(16, dtype=torch.bfloat16, device="cuda")
