@@ -55,6 +55,7 @@ def test_workspace_size_grows_with_blocks(lib_path):
     s.num_ctas = 400
     b = lib.rgd_prefix_decode_attn_workspace_size(ctypes.byref(s))
     # tickets for 128 jobs + (ctas + jobs - 1) partial slots of 20 queries x (128 + 2) floats
-    assert b - a == 300 * 20 * 128 * 4 + 300 * 20 * 8
+    grow = 300 * 20 * 128 * 4 + 300 * 20 * 8
+    assert grow <= b - a < grow + 512  # each region is padded to 256 bytes
     s.reserved = 1
     assert lib.rgd_prefix_decode_attn_workspace_size(ctypes.byref(s)) == 0
