@@ -281,7 +281,7 @@ def run_ours(args):
         with torch.cuda.graph(g_hg, stream=stream):
             head_gate_call()
         torch.cuda.synchronize()
-    launches_per_step = 4  # attention, sample head, gate-state reset, gate
+    launches_per_step = 5  # attention, split-job merge, sample head, gate-state reset, gate
 
     def one_step(ev):
         flush.fill_(1)

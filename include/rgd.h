@@ -117,10 +117,11 @@ size_t rgd_prefix_decode_attn_workspace_size(const rgd_attn_shape* shape);
  *   softmax_scale      > 0 (1/sqrt(D) for standard attention)
  *   out                bf16 [R, Hq, D]; lse float [R, Hq] or NULL
  *   workspace          device memory of rgd_prefix_decode_attn_workspace_size()
- *                      bytes, 256-byte aligned, ZERO-FILLED before its first use;
- *                      a successful call leaves it zero-filled again (re-zero it
- *                      after a call that reported a device error).  Calls that
- *                      share a workspace must not overlap in time.
+ *                      bytes, 256-byte aligned, contents arbitrary (a call
+ *                      reads only what it wrote there).  Calls that share a
+ *                      workspace must not overlap in time.
+ * Two kernels run on `stream`: the attention kernel and a small merge of the
+ * jobs that were split across blocks.
  * A group with prompt_len 0 and a row with suffix_len 0 are valid; a row with
  * neither gets out = 0, lse = -inf.  Page ids outside [0, num_pages) read as
  * zeros and set RGD_DEV_BAD_PAGE.  Lengths beyond the table are rejected on the
@@ -135,7 +136,7 @@ int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf16* q,
 
 /* Allocation-free form of rgd_prefix_decode_attn (the paper has no counterpart;
  * this is a deployment convenience).  Same arguments and results, minus the
- * workspace: the split partials and merge tickets live in one fixed 8 MiB device
+ * workspace: the split partials live in one fixed 8 MiB device
  * array inside the library (one per device, held by every process that loads the
  * library until it exits).  It is for callers that cannot call cudaMalloc: for
  * example a serving engine whose KV-cache manager has already reserved the free
@@ -147,10 +148,9 @@ int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf16* q,
  *   - The first call on a device looks up the array's device address (once per
  *     device, with that device current); make that first call before any stream
  *     capture.
- *   - Each call clears the tickets with cudaMemsetAsync on `stream`; nothing is
- *     allocated.  Every call shares the one array and it keeps the last call's
- *     contents, so calls that overlap on the GPU (other streams, other threads)
- *     race: serialise them. */
+ *   - Nothing is allocated or cleared: a call reads only scratch values that it
+ *     wrote itself.  Every call shares the one array, so calls that overlap on
+ *     the GPU (other streams, other threads) race: serialise them. */
 int rgd_prefix_decode_attn_noalloc(const rgd_attn_shape* shape, const rgd_bf16* q,
                                    const rgd_bf16* k_pages, const rgd_bf16* v_pages,
                                    const int32_t* prompt_block_table, const int32_t* prompt_len,

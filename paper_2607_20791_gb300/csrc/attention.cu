@@ -1,4 +1,4 @@
-// Shared-prefix decode attention: persistent, balanced, one pass over the KV.
+// Shared-prefix decode attention on the 5th-generation tensor cores.
 //
 // Sec. 3 reuses the prompt KV cache across the greedy probe and the high-
 // temperature sampling stage.  Here that reuse is explicit: for every prompt
@@ -11,17 +11,39 @@
 // HBM exactly once.
 //
 // Work distribution.  The jobs' page lists are laid end to end (job-major) and
-// the grid's persistent CTAs (one per SM) each take an equal contiguous range of
-// pages.  Inside a CTA a producer warp streams its pages' 16-token K/V tiles into
-// a shared-memory ring with 2-D TMA loads (128-byte swizzle), across job
-// boundaries, paced by full/empty mbarriers whose waits are all bounded.  Fifteen
-// consumer warps own (query tile of 16, token slice) pairs and run S = Q K^T and
-// O += P V on bf16 tensor-core MMAs with an online softmax in fp32.  At the end
-// of each job piece the token slices are combined in shared memory; a job that
-// lies inside one CTA is written out directly, a job split across CTAs leaves a
-// partial (o, m, l) in workspace slot (cta + job) -- distinct for every piece,
-// since CTA ranges are ordered like the jobs -- and the last piece to finish
-// (atomic ticket, no waiting) merges the partials by log-sum-exp.
+// the grid's persistent blocks (one per SM) each take an equal contiguous range
+// of pages.  A job split across blocks leaves a partial (o, m, l) in workspace
+// slot (block + job) -- distinct for every piece, since block ranges are ordered
+// like the jobs -- and a second, small kernel merges each split job's partials
+// by log-sum-exp (Sec. 3's shared-prefix split is the same identity).
+//
+// Inside a block (576 threads) the tensor memory holds Q, S / P and O, so the
+// tensor cores read only K and V from shared memory -- the bytes that come from
+// HBM:
+//   * warp 16 (producer) streams the pages, four to a group, into a ring of
+//     group slots with 3-D TMA boxes (128-byte swizzle): each K tile lands as
+//     two 2 KiB halves in a half-major, group-contiguous block, so that one MMA
+//     covers all the group's tokens (an MMA costs ~50 cycles to issue whatever
+//     its N, so the number of MMAs, not their size, is what counts), each V
+//     tile as one box; every lane issues its own page, since one issuing
+//     thread is copy-rate bound;
+//   * warp 17 allocates the tensor memory and its lane 0 issues every MMA: for a
+//     group of up to 4 pages, S = Q K^T (A = Q from TMEM, M = 128 query rows,
+//     N = 16 x pages) into one of three S/P buffers, and, once the
+//     softmax warps have turned S into bf16 P in place, O += P V per page (A = P
+//     from TMEM, N = the head dimension, V read MN-major from its tile); one
+//     commit after the group's PV hands its slot back to the producer;
+//   * warps 0-15: warp w owns TMEM lanes 32(w%4)..+31 (query rows) and page w/4
+//     of the group, so every thread handles the 16 scores of one row and one
+//     page: the masks, the group's row max (exchanged through shared memory),
+//     the online softmax in fp32 (the running max is only moved, and O rescaled
+//     in TMEM, when a row's max grows by more than 2^8) and its 16 bf16 P values;
+//     they also write Q into TMEM, and at the end of a job piece the four warps
+//     of a lane quarter each read a quarter of O's columns and write the output
+//     or the partial.  Warps whose lane quarter holds only padding rows (>= the
+//     job's query count) sit out.
+// Every wait on an mbarrier is bounded; a timeout is reported in the status
+// word and every role stops.
 #include <cudaTypedefs.h>
 
 #include <cmath>
@@ -34,12 +56,26 @@ namespace rgd {
 namespace {
 
 constexpr int kPage = 16;
-constexpr int kCWarps = 15;                  // consumer warps (16 warps in all: <= 128 registers each)
-constexpr int kCThreads = kCWarps * 32;
-constexpr int kAttnThreads = kCThreads + 32;  // + one producer warp
-constexpr int kMaxStages = 16;
-constexpr int kMaxQueries = 128;  // rows_per_group * Hq / Hkv
-constexpr int kSmemLimit = 226 * 1024;  // dynamic part; the kernel's static shared memory needs the rest
+constexpr int kSoftWarps = 16;                // warps 0-15: softmax / epilogue
+constexpr int kSoftThreads = kSoftWarps * 32;
+constexpr int kProducerWarp = 16;
+constexpr int kMmaWarp = 17;
+constexpr int kAttnThreads = 18 * 32;
+constexpr int kGroupPages = 4;                // pages per S / P buffer (64 tokens)
+constexpr int kMaxSlots = 8;                  // ring slots, one page group each
+constexpr int kSPBufs = 3;                    // S / P buffers in TMEM
+constexpr int kRows = 128;                    // MMA M: query rows per job
+constexpr int kMaxQueries = kRows;            // rows_per_group * Hq / Hkv
+constexpr int kTmemCols = 512;
+constexpr int kOCol = 0;                      // O: columns [0, D)
+constexpr int kSPCol = 128;                   // S / P buffers: 64 columns each
+constexpr int kQCol = kSPCol + kSPBufs * 64;  // Q buffers: D/2 columns each (two bf16 per column)
+// V as the MN-major B operand of PV: the two 64-column halves of a page tile are
+// MN-direction swizzle atoms 2048 B apart, the two 8-token groups K-direction
+// atoms 1024 B apart.
+constexpr uint32_t kVLbo = 2048, kVSbo = 1024;
+constexpr float kRescaleLog2 = 8.f;           // lazy rescale threshold (factor 256)
+constexpr int kSmemLimit = 226 * 1024;        // dynamic part; static shared memory needs the rest
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
@@ -54,64 +90,52 @@ struct AttnParams {
   float* lse;
   float* slot_o;    // [(C + J - 1) * nq, D]
   float2* slot_ml;  // [(C + J - 1) * nq]
-  int32_t* ticket;  // [J]
+  int32_t* gpre_ws; // [G + 1] page-count prefix, written by block 0 for the merge
   int32_t* dev_status;
   int32_t G, rpg, Hq, Hkv, gq, num_pages, max_pp, max_sp;
-  int32_t nq, n_mt, TS, nst, C;
+  int32_t nq, nslots, C;
   float scale_log2;
 };
 
-// Shared-memory carve-up (identical on host and device).
+// Shared-memory carve-up (identical on host and device).  The ring is 1024-byte
+// aligned: the 128-byte swizzle repeats every 8 rows of 128 bytes.
 struct SmemLayout {
-  int ring, q, acc, ml, gpre, desc, total;
+  int ring, red, gpre, gact, desc, total;
 };
 
 __host__ __device__ inline int align_up(int x, int a) { return (x + a - 1) / a * a; }
 
+// One ring slot holds a page group: its K tiles half-major and group-contiguous
+// ([D/64 halves][4 pages][16 rows][128 B], so that one MMA reads the whole
+// group's K for a 16-wide slice of the head dimension), then its V tiles
+// ([4 pages][D/64 halves][16 rows][128 B]).
 template <int D>
-__host__ __device__ inline SmemLayout smem_layout(int nst, int n_mt, int TS, int G) {
-  SmemLayout L;
-  L.ring = 0;
-  L.q = nst * 2 * kPage * D * 2;
-  L.acc = align_up(L.q + n_mt * 16 * (D * 2 + 16), 16);
-  L.ml = align_up(L.acc + n_mt * 16 * (D + 4) * 4, 16);
-  L.gpre = align_up(L.ml + TS * n_mt * 16 * 8, 16);
-  L.desc = align_up(L.gpre + (G + 1) * 4, 16);
-  L.total = align_up(L.desc + nst * 4, 16) + 1024;  // + alignment slack for the 1024-B ring base
-  return L;
+__host__ __device__ constexpr int slot_bytes() {
+  return 2 * kGroupPages * kPage * D * 2;
 }
 
-// Byte offset of (token t, 16-byte chunk c) in a page tile loaded as 64-column
-// boxes with the 128-byte swizzle (chunk index XOR row index mod 8).
-__device__ __forceinline__ uint32_t swz(uint32_t tile, int t, int c) {
-  return tile + ((c >> 3) << 11) + (t << 7) + ((((c & 7) ^ (t & 7))) << 4);
+template <int D>
+__host__ __device__ inline SmemLayout smem_layout(int nslots, int G) {
+  SmemLayout L;
+  L.ring = 0;
+  L.red = nslots * slot_bytes<D>();
+  // row-max exchange (2 buffers), row-sum exchange, per-lane (m, l), O staging (2 buffers)
+  L.gpre = L.red + (3 * 4 * kRows + 2 * kRows + 2 * 4 * 32 * 16) * 4;
+  L.gact = align_up(L.gpre + (G + 1) * 4, 16);
+  L.desc = align_up(L.gact + G * 4, 16);
+  L.total = align_up(L.desc + nslots * kGroupPages * 4, 16) + 1024;  // + slack for the 1024-byte aligned base
+  return L;
 }
 
 __device__ __forceinline__ void flag(int32_t* status, int32_t bit) {
   if (status) atomicOr(status, bit);
 }
 
-__device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kCThreads) : "memory"); }
-
 __device__ __forceinline__ bool row_on(const AttnParams& p, int r) {
   return p.row_active == nullptr || p.row_active[r] != 0;
 }
 
 __device__ __forceinline__ int clamp_len(int n, int max_pages) { return n < 0 ? 0 : min(n, max_pages * kPage); }
-
-// Pages of one (group, kv head) job: the prompt pages if any row of the group is
-// active, plus the suffix pages of every active row.
-__device__ int group_pages(const AttnParams& p, int g) {
-  bool any = false;
-  int sp = 0;
-  for (int i = 0; i < p.rpg; ++i) {
-    const int r = g * p.rpg + i;
-    if (!row_on(p, r)) continue;
-    any = true;
-    sp += (clamp_len(p.suffix_len[r], p.max_sp) + kPage - 1) / kPage;
-  }
-  return any ? (clamp_len(p.prompt_len[g], p.max_pp) + kPage - 1) / kPage + sp : 0;
-}
 
 struct Job {
   int g, h, n;      // group, kv head, pages
@@ -148,51 +172,109 @@ __device__ Job next_job(const AttnParams& p, const int32_t* gpre, Job j) {
   return j;
 }
 
-// CTA whose page range contains global page x (ranges [floor(cT/C), floor((c+1)T/C))).
+// Block whose page range contains global page x (ranges [floor(cT/C), floor((c+1)T/C))).
 __device__ __forceinline__ int cta_of(int64_t x, int64_t T, int C) { return (int)(((x + 1) * C - 1) / T); }
+
+// Bounded wait that also gives up as soon as another role has given up.
+__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag) {
+  if (*abort_flag) return false;
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 63u) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        *abort_flag = 1;
+        return false;
+      }
+    }
+  }
+}
 
 template <int D>
 __global__ void __launch_bounds__(kAttnThreads, 1)
-    attn_persistent_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
-                           const AttnParams p) {
-  constexpr int kTile = kPage * D * 2;
-  constexpr int kStage = 2 * kTile;
-  constexpr int kQStride = D * 2 + 16;
-  constexpr int kAccStride = D + 4;
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                   const AttnParams p) {
+  constexpr int kTile = kPage * D * 2;      // one K or V page-head tile
+  constexpr int kStage = 2 * kTile;         // bytes one page brings in
+  constexpr int kHalves = D / 64;
+  constexpr int kSlot = slot_bytes<D>();
+  constexpr int kVOff = kGroupPages * kTile;  // V tiles within a slot
+  constexpr uint32_t kIdescPV = idesc_bf16_f32(kRows, D, 0, 1);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const SmemLayout L = smem_layout<D>(p.nst, p.n_mt, p.TS, p.G);
+  const SmemLayout L = smem_layout<D>(p.nslots, p.G);
   int32_t* gpre = reinterpret_cast<int32_t*>(smem + L.gpre);
   uint32_t* descs = reinterpret_cast<uint32_t*>(smem + L.desc);
-  uint8_t* qs = smem + L.q;
-  float* acc = reinterpret_cast<float*>(smem + L.acc);
-  float2* mls = reinterpret_cast<float2*>(smem + L.ml);
-  __shared__ uint64_t full_bar[kMaxStages], empty_bar[kMaxStages];
-  __shared__ int32_t s_abort, s_piece_abort, s_issued, s_last, s_wsum[kAttnThreads / 32];
+  __shared__ uint64_t full_bar[kMaxSlots], empty_bar[kMaxSlots];
+  __shared__ uint64_t s_full[kSPBufs], p_full[kSPBufs], p_empty[kSPBufs], q_full[2], q_empty[2], o_free, mma_done;
+  __shared__ int32_t s_abort, s_issued, s_wsum[kAttnThreads / 32];
+  __shared__ uint32_t s_tmem;
+  volatile int32_t* abort_flag = &s_abort;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int c = blockIdx.x;
-  const int nst = p.nst;
+  const int ns = p.nslots;
+  const uint32_t sbase = smem_u32(smem);
+  // The queries fill qpc TMEM lane quarters and are held R times; the softmax
+  // warps of unused quarters sit out, and the barriers count the active ones.
+  const int qpc = (p.nq + 31) / 32;         // lane quarters one copy of the queries spans
+  const int R = 4 / qpc;                    // copies of the queries in the 128 lanes
+  const int W = kGroupPages / R;            // softmax warps per quarter (pages per copy and group)
+  const int n_act = R * qpc * W;            // active softmax warps
 
   if (tid == 0) {
-    for (int i = 0; i < nst; ++i) {
-      mbar_init(&full_bar[i], 1);
-      mbar_init(&empty_bar[i], p.n_mt);
+    for (int i = 0; i < ns; ++i) {
+      mbar_init(&full_bar[i], kGroupPages);  // one arrival per page position (absent pages of a short group too)
+      mbar_init(&empty_bar[i], 1);           // released by an MMA commit once the group's PV is done
     }
+    for (int i = 0; i < kSPBufs; ++i) {
+      mbar_init(&s_full[i], 1);
+      mbar_init(&p_full[i], n_act);
+      mbar_init(&p_empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&q_full[i], n_act);
+      mbar_init(&q_empty[i], 1);
+    }
+    mbar_init(&o_free, n_act);
+    mbar_init(&mma_done, 1);
     s_abort = 0;
     s_issued = 0;
     fence_mbar_init();
   }
-  // ---- page counts per group and their exclusive prefix sum (every CTA) ----
-  for (int g = tid; g < p.G; g += kAttnThreads) gpre[g + 1] = group_pages(p, g);
+  if (warp == kMmaWarp) {
+    tmem_alloc(&s_tmem, kTmemCols);
+    tmem_relinquish();
+  }
+  // ---- page counts per group and their exclusive prefix sum (every block) ----
+  // Rows are read in parallel (one global-memory latency, not one per row).
+  int32_t* gact = reinterpret_cast<int32_t*>(smem + L.gact);
+  for (int g = tid; g < p.G; g += kAttnThreads) {
+    gpre[g + 1] = 0;
+    gact[g] = 0;
+  }
   if (tid == 0) gpre[0] = 0;
+  __syncthreads();
+  for (int r = tid; r < p.G * p.rpg; r += kAttnThreads) {
+    if (!row_on(p, r)) continue;
+    atomicAdd(&gpre[r / p.rpg + 1], (clamp_len(p.suffix_len[r], p.max_sp) + kPage - 1) / kPage);
+    atomicOr(&gact[r / p.rpg], 1);
+  }
+  __syncthreads();
+  for (int g = tid; g < p.G; g += kAttnThreads)
+    gpre[g + 1] = gact[g] ? gpre[g + 1] + (clamp_len(p.prompt_len[g], p.max_pp) + kPage - 1) / kPage : 0;
   if (c == 0) {
     for (int g = tid; g < p.G; g += kAttnThreads)
       if (p.prompt_len[g] < 0 || p.prompt_len[g] > p.max_pp * kPage) flag(p.dev_status, RGD_DEV_BAD_PAGE);
     for (int r = tid; r < p.G * p.rpg; r += kAttnThreads)
       if (p.suffix_len[r] < 0 || p.suffix_len[r] > p.max_sp * kPage) flag(p.dev_status, RGD_DEV_BAD_PAGE);
   }
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
   {
     const int E = (p.G + kAttnThreads - 1) / kAttnThreads;
     const int lo = 1 + tid * E, hi = min(p.G + 1, lo + E);
@@ -222,6 +304,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     }
   }
   __syncthreads();
+  if (c == 0)
+    for (int g = tid; g <= p.G; g += kAttnThreads) p.gpre_ws[g] = gpre[g];
   const int64_t T = (int64_t)p.Hkv * gpre[p.G];
   // pages are divided over Ceff = min(C, T) blocks so that every working block
   // has at least one page (a job's pieces are then exactly the blocks first..last)
@@ -229,30 +313,37 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int64_t b = c < Ceff ? (int64_t)c * T / Ceff : T;
   const int64_t e = c < Ceff ? (int64_t)(c + 1) * T / Ceff : T;
 
-  if (warp == kCWarps) {
+  if (warp == kProducerWarp) {
     // ============================ producer ============================
-    // The warp resolves 32 pages at a time, one per lane (job by binary search
-    // in shared memory, then the block-table entry), so the global-memory
-    // latency of the page lookups is paid once per 32 pages, and every lane then
-    // issues its own page's two 4 KiB copies: the copy rate of a single issuing
-    // thread, not HBM, is what limits a one-thread producer.
+    // The warp resolves 32 consecutive pages at a time, one per lane (job by
+    // binary search in shared memory, then the block-table entry).  Then, group
+    // by group, the lane holding a group's first page waits for its slot (group
+    // g of this block goes to slot g % nslots) and every lane of the group
+    // issues its own page's copies: K as two 2 KiB halves into the group's
+    // half-major K block, V as one box.  Groups go in order, so the slot wait
+    // (for the PV of the group nslots back, issued after the QK of the group
+    // after it) never depends on a page not yet issued.
     if (b < e) {
       if (lane == 0) {
         prefetch_tensormap(&tmK);
         prefetch_tensormap(&tmV);
       }
       const uint64_t pol = policy_evict_first();
-      bool aborted = false;
-      // A batch holds at most one page per ring slot, so each lane's parity wait
-      // on its slot is never more than one phase ahead of the consumers.
-      const int nb = min(32, nst);
-      for (int64_t xb = b; xb < e && !aborted; xb += nb) {
+      int gbase = 0;  // groups started before xb
+      int64_t xb = b;
+      while (xb < e) {
         const int64_t x = xb + lane;
-        const bool mine = lane < nb && x < e;
-        int32_t page = -1, tok = 0, rowsel = -1, hh = 0;
-        if (mine) {
+        const bool valid = x < e;
+        int32_t page = -1, tok = 0, rowsel = -1, hh = 0, jpos = 0, ng = 0;
+        if (valid) {
           const Job jb = job_at(p, gpre, x);
           const int k = (int)(x - jb.start);
+          // this block's piece of the job starts at max(b, job start); groups restart there
+          const int64_t pstart = max(b, jb.start);
+          const int kin = (int)(x - pstart);
+          const int npiece = (int)(min(e, jb.start + jb.n) - pstart);
+          jpos = kin % kGroupPages;
+          ng = min(kGroupPages, npiece - (kin - jpos));
           const int plen = clamp_len(p.prompt_len[jb.g], p.max_pp);
           const int ppg = (plen + kPage - 1) / kPage;
           hh = jb.h;
@@ -275,312 +366,479 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             }
           }
         }
-        // every lane issues its own page: up to 32 copy streams in flight
-        int stop = 0;
-        if (mine) {
-          const int64_t li = x - b;
-          const int slot = (int)(li % nst);
-          if (li >= nst && !mbar_wait(&empty_bar[slot], (uint32_t)((li / nst) - 1) & 1u)) s_abort = 1;
-          if (*(volatile int32_t*)&s_abort) {
+        const bool start = valid && jpos == 0;
+        const uint32_t starts = __ballot_sync(0xffffffffu, start);
+        const uint32_t le = 0xffffffffu >> (31 - lane);
+        const int gidx = gbase + __popc(starts & le) - 1;  // lane 0 may continue the last round's group
+        const int g0 = __shfl_sync(0xffffffffu, gidx, 0);
+        const int g1 = __shfl_sync(0xffffffffu, gidx, 31 - __clz(__ballot_sync(0xffffffffu, valid)));
+        const int gs = gidx % ns;
+        bool aborted = false;
+        for (int gq = g0; gq <= g1; ++gq) {
+          const bool in = valid && gidx == gq;
+          int stop = 0;
+          if (in && start && gq >= ns &&
+              !wait_or_abort(&empty_bar[gs], (uint32_t)((gq / ns) - 1) & 1u, abort_flag))
             stop = 1;
-          } else {
+          if (__any_sync(0xffffffffu, stop != 0)) {
+            aborted = true;
+            break;
+          }
+          if (in) {
             int32_t y = -2 * kPage;  // fully out of bounds: the TMA fills zeros
             if (page >= 0 && page < p.num_pages) y = (page * p.Hkv + hh) * kPage;
             else flag(p.dev_status, RGD_DEV_BAD_PAGE);
-            descs[slot] = (uint32_t)tok | ((uint32_t)(rowsel & 0xffff) << 16);
-            uint8_t* kt = smem + slot * kStage;
-            mbar_arrive_expect_tx(&full_bar[slot], kStage);
-            tma_load_3d_hint(kt, &tmK, &full_bar[slot], 0, y, 0, pol);
-            tma_load_3d_hint(kt + kTile, &tmV, &full_bar[slot], 0, y, 0, pol);
-            atomicMax(&s_issued, (int)(li + 1));
+            descs[gs * kGroupPages + jpos] = (uint32_t)tok | ((uint32_t)(rowsel & 0xffff) << 16);
+            uint8_t* sl = smem + gs * kSlot;
+            mbar_arrive_expect_tx(&full_bar[gs], kStage);
+            if (jpos == ng - 1 && ng < kGroupPages) mbar_arrive_cnt(&full_bar[gs], kGroupPages - ng);
+#pragma unroll
+            for (int hf = 0; hf < kHalves; ++hf)
+              tma_load_3d_hint(sl + hf * (kGroupPages * 2048) + jpos * 2048, &tmK, &full_bar[gs], 0, y, hf, pol);
+            tma_load_3d_hint(sl + kVOff + jpos * kTile, &tmV, &full_bar[gs], 0, y, 0, pol);
+            if (start) s_issued = gq + 1;
           }
         }
-        aborted = __any_sync(0xffffffffu, stop != 0);
+        if (aborted) break;
+        gbase += __popc(starts);
+        xb += 32;
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    // ============================ MMA issue ===========================
+    // B descriptors are formed once; an MMA's B differs from the ring base only
+    // in the start-address field (byte offset / 16).
+    if (lane == 0 && b < e) {
+      const uint64_t k_d = smem_desc(sbase, 1024, 1024, 2);
+      const uint64_t v_d = smem_desc(sbase, D == 128 ? kVLbo : 1024, D == 128 ? kVSbo : 1024, 2);
+      int gi = 0, pc = 0;
+      // the previous group's PV waits until the next group's QK is issued
+      int pv_gi = -1, pv_n = 0, pv_first = 0, pv_pc = 0;
+      bool ok = true;
+      auto issue_pv = [&]() {
+        const int pb = pv_gi % kSPBufs;
+        const int gs = pv_gi % ns;
+        if (!wait_or_abort(&p_full[pb], (uint32_t)(pv_gi / kSPBufs) & 1u, abort_flag)) return false;
+        if (pv_first && pv_pc >= 1 && !wait_or_abort(&o_free, (uint32_t)(pv_pc - 1) & 1u, abort_flag)) return false;
+        tc_fence_after();
+#pragma unroll
+        for (int j = 0; j < kGroupPages; ++j) {
+          if (j < pv_n)
+            umma_bf16_tmem_a(tmem + kOCol, tmem + kSPCol + pb * 64 + j * 8,
+                             v_d + (uint64_t)((gs * kSlot + kVOff + j * kTile) >> 4), kIdescPV,
+                             (pv_first && j == 0) ? 0u : 1u);
+        }
+        umma_commit(&p_empty[pb]);
+        umma_commit(&empty_bar[gs]);  // the slot's K and V are no longer read
+        return true;
+      };
+      Job cur = job_at(p, gpre, b);
+      int64_t x0 = b;
+      while (ok && x0 < e) {
+        const int n_in = (int)(min(e, cur.start + cur.n) - x0);
+        const int qb = pc & 1;
+        if (!wait_or_abort(&q_full[qb], (uint32_t)(pc >> 1) & 1u, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t qa = tmem + kQCol + qb * (D / 2);
+        for (int k0 = 0; k0 < n_in; k0 += kGroupPages) {
+          const int ng = min(kGroupPages, n_in - k0);
+          const int sb = gi % kSPBufs;
+          const int gs = gi % ns;
+          if (!wait_or_abort(&full_bar[gs], (uint32_t)(gi / ns) & 1u, abort_flag)) {
+            ok = false;
+            break;
+          }
+          // the S / P buffer is free once the PV of the group that used it last is done
+          if (gi >= kSPBufs && !wait_or_abort(&p_empty[sb], (uint32_t)((gi / kSPBufs) - 1) & 1u, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t idesc_qk = idesc_bf16_f32(kRows, kPage * ng, 0, 0);
+          const uint64_t kg = k_d + (uint64_t)((gs * kSlot) >> 4);
+          const uint32_t dcol = tmem + kSPCol + sb * 64;
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk)
+            umma_bf16_tmem_a(dcol, qa + kk * 8,
+                             kg + (uint64_t)(((kk >> 2) * (kGroupPages * 2048) + (kk & 3) * 32) >> 4), idesc_qk,
+                             kk > 0 ? 1u : 0u);
+          umma_commit(&s_full[sb]);
+          if (k0 + ng == n_in) umma_commit(&q_empty[qb]);
+          if (pv_gi >= 0 && !issue_pv()) {
+            ok = false;
+            break;
+          }
+          pv_gi = gi;
+          pv_n = ng;
+          pv_first = (k0 == 0);
+          pv_pc = pc;
+          ++gi;
+        }
+        if (ok && pv_gi >= 0 && !issue_pv()) ok = false;
+        pv_gi = -1;
+        ++pc;
+        x0 += n_in;
+        if (x0 < e) cur = next_job(p, gpre, cur);
       }
     }
   } else {
-    // ============================ consumers ===========================
-    const int n_mt = p.n_mt, TS = p.TS, nq = p.nq, gq = p.gq;
-    const int mt = warp % n_mt, ts = warp / n_mt;
-    const bool busy = warp < n_mt * TS;
-    const int col = 2 * (lane & 3);
-    const int qi0 = mt * 16 + (lane >> 2), qi1 = qi0 + 8;
-    const int rloc0 = qi0 < nq ? qi0 / gq : -2, rloc1 = qi1 < nq ? qi1 / gq : -2;
-    const uint32_t ring = smem_u32(smem);
+    // ============================ softmax / epilogue =================
+    // The nq query rows span qpc = ceil(nq / 32) TMEM lane quarters, so R = 4 / qpc
+    // copies of them fit in the 128 lanes (Q is written R times; S costs the
+    // same MMAs either way).  Copy c handles pages c, c + R, ... of every group
+    // with an online softmax of its own, and W = 4 / R warps of each of its
+    // quarters (one page each) share that copy's running max; its P is zero in
+    // the other copies' page columns, so O in its lanes sums its own pages only.
+    // The copies are merged by log-sum-exp at the end of the piece.  For nq <= 32
+    // each page of a group is thus handled on its own SM sub-partition (a warp
+    // can only reach its own lane quarter) and no warp waits for another between
+    // groups.
+    const int nq = p.nq, gq = p.gq;
+    const int qd = warp & 3, pj = warp >> 2;  // TMEM lane quarter; warp within the quarter
+    const int cp = qd / qpc, rb = qd % qpc;   // copy; row block of the queries
+    const bool active = cp < R && pj < W;
+    const int jp = cp + pj * R;               // this warp's page within a group
+    const int n_athr = n_act * 32;
+    auto soft_sync = [&]() { asm volatile("bar.sync 1, %0;" ::"r"(n_athr) : "memory"); };
+    const int r = rb * 32 + lane;              // this thread's query
+    const int rloc = r < nq ? r / gq : -2;     // its row within the group (suffix pages are per row)
+    const int tlane = qd * 32 + lane;          // its TMEM lane
+    const uint32_t tl = tmem + ((uint32_t)(qd * 32) << 16);
+    float* rmax = reinterpret_cast<float*>(smem + L.red);  // [2][4][128] page-slot maxima
+    float* rsum = rmax + 2 * 4 * kRows;                    // [4][128] page-slot row sums
+    float2* mlx = reinterpret_cast<float2*>(rsum + 4 * kRows);  // [128] (m, l) of each lane
+    float4* stage = reinterpret_cast<float4*>(mlx + kRows);     // [2][<= 4 * 32 * 4] O columns of copies >= 1
+    const int ocols = D / W;                   // O columns read / rescaled by each warp of a quarter
+    const int qcols = (D / 2) / W;             // Q columns (bf16 pairs) written by each warp of a quarter
+    // warp-uniform bounded wait (TMEM loads and stores that follow are warp-collective)
+    auto wwait = [&](uint64_t* bar, uint32_t parity, volatile int32_t* flag) {
+      return __all_sync(0xffffffffu, wait_or_abort(bar, parity, flag));
+    };
 
     // jobs with no pages at all (empty prompt and suffixes, some row active)
     for (int j = c; j < p.G * p.Hkv; j += p.C) {
       const int g = j / p.Hkv, h = j % p.Hkv;
       if (gpre[g + 1] != gpre[g]) continue;
-      for (int idx = tid; idx < nq * D; idx += kCThreads) {
+      for (int idx = tid; idx < nq * D; idx += kSoftThreads) {
         const int i = idx / D, d = idx % D;
-        const int r = g * p.rpg + i / gq, hq = h * gq + i % gq;
-        if (!row_on(p, r)) continue;
-        p.out[((int64_t)r * p.Hq + hq) * D + d] = __float2bfloat16(0.f);
-        if (d == 0 && p.lse) p.lse[(int64_t)r * p.Hq + hq] = -INFINITY;
+        const int rr = g * p.rpg + i / gq, hq = h * gq + i % gq;
+        if (!row_on(p, rr)) continue;
+        p.out[((int64_t)rr * p.Hq + hq) * D + d] = __float2bfloat16(0.f);
+        if (d == 0 && p.lse) p.lse[(int64_t)rr * p.Hq + hq] = -INFINITY;
       }
     }
 
-    float o[D / 8][4];
+    // These warps never leave their loops early: the loop structure is the same
+    // for all of them, so every named barrier is reached even after an abort
+    // (waits then return at once and the work is skipped).
+    int gi = 0, pc = 0;
+    bool ok = true;
     Job cur;
-    if (b < e) cur = job_at(p, gpre, b);
-    int64_t x0 = b;
+    if (b < e && active) cur = job_at(p, gpre, b);
+    int64_t x0 = active ? b : e;
     while (x0 < e) {
-      const int64_t pe = min(e, cur.start + cur.n);
+      const int n_in = (int)(min(e, cur.start + cur.n) - x0);
       const int j = cur.g * p.Hkv + cur.h;
-      // ---- queries of the job -> shared memory; zero the combine buffer ----
-      constexpr int kChunks = D / 8;
-      for (int idx = tid; idx < n_mt * 16 * kChunks; idx += kCThreads) {
-        const int i = idx / kChunks, ch = idx % kChunks;
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (i < nq) {
-          const int r = cur.g * p.rpg + i / gq, hq = cur.h * gq + i % gq;
-          v = __ldg(reinterpret_cast<const uint4*>(p.q + ((int64_t)r * p.Hq + hq) * D) + ch);
+      const int qb = pc & 1;
+      // ---- this warp's share of its rows' queries -> Q buffer in TMEM ----
+      if (pc >= 2 && ok && !wwait(&q_empty[qb], (uint32_t)((pc >> 1) - 1) & 1u, abort_flag)) ok = false;
+      if (ok) {
+        constexpr int kQChunk = 8;    // uint4 loads in flight (32 registers)
+        const int nld = qcols / 4;    // uint4 loads of this warp's share
+        const bool qrow = r < nq;
+        const uint4* src = nullptr;
+        if (qrow) {
+          const int rr = cur.g * p.rpg + r / gq, hq = cur.h * gq + r % gq;
+          src = reinterpret_cast<const uint4*>(p.q + ((int64_t)rr * p.Hq + hq) * D) + pj * nld;
         }
-        *reinterpret_cast<uint4*>(qs + i * kQStride + ch * 16) = v;
+        const uint32_t qcol = kQCol + qb * (D / 2) + pj * qcols;
+#pragma unroll 1
+        for (int t0 = 0; t0 < nld; t0 += kQChunk) {
+          uint4 qv[kQChunk];
+#pragma unroll
+          for (int t = 0; t < kQChunk; ++t)
+            qv[t] = (qrow && t0 + t < nld) ? __ldg(src + t0 + t) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+          for (int t = 0; t < kQChunk / 2; ++t) {
+            if (t0 + 2 * t < nld) {
+              const uint32_t v8[8] = {qv[2 * t].x,     qv[2 * t].y,     qv[2 * t].z,     qv[2 * t].w,
+                                      qv[2 * t + 1].x, qv[2 * t + 1].y, qv[2 * t + 1].z, qv[2 * t + 1].w};
+              tmem_st8(tl + qcol + (t0 / 2 + t) * 8, v8);
+            }
+          }
+        }
+        tmem_st_wait();
       }
-      for (int idx = tid; idx < n_mt * 16 * kAccStride; idx += kCThreads) acc[idx] = 0.f;
-      consumer_sync();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&q_full[qb]);
 
-      float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-#pragma unroll
-      for (int i = 0; i < D / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-      if (busy) {
-        const uint32_t qbase =
-            smem_u32(qs) + (mt * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * kQStride + (lane >> 4) * 16;
-        const int kt_t = (lane & 7) + ((lane >> 4) & 1) * 8, kt_c = (lane >> 3) & 1;
-        const int vt_t = (lane & 7) + ((lane >> 3) & 1) * 8, vt_c = lane >> 4;
-        const int lb = (int)(x0 - b), le = (int)(pe - b);
-        int li = lb + ((ts - lb % TS) + TS) % TS;
-        int slot = li % nst;  // ring slot and phase advance incrementally (TS divides nst)
-        uint32_t phase = (uint32_t)(li / nst) & 1u;
-        for (; li < le; li += TS) {
-          if (*(volatile int32_t*)&s_abort) break;
-          if (!mbar_wait(&full_bar[slot], phase)) {
-            s_abort = 1;
-            break;
+      float m_used = -INFINITY, l = 0.f;  // m_used is shared by the W warps of a quarter; l is per warp
+      for (int k0 = 0; k0 < n_in; k0 += kGroupPages) {
+        const int ng = min(kGroupPages, n_in - k0);
+        const int sb = gi % kSPBufs, gs = gi % ns;
+        if (ok && !wwait(&s_full[sb], (uint32_t)(gi / kSPBufs) & 1u, abort_flag)) ok = false;
+        const bool has = ok && jp < ng;
+        tc_fence_after();
+        int tok = 0, sel = -1;
+        if (has) {
+          // this page's descriptor; the producer's write is ordered by the full barrier
+          if (wwait(&full_bar[gs], (uint32_t)(gi / ns) & 1u, abort_flag)) {
+            const uint32_t dsc = descs[gs * kGroupPages + jp];
+            tok = (int)(dsc & 0xffffu);
+            sel = (int)(int16_t)(dsc >> 16);
+          } else {
+            ok = false;
           }
-          const uint32_t desc = descs[slot];
-          const int tok = (int)(desc & 0xffffu);
-          const int rowsel = (int)(int16_t)(desc >> 16);
-          const bool ok0 = rowsel < 0 || rloc0 == rowsel, ok1 = rowsel < 0 || rloc1 == rowsel;
-          const uint32_t ktile = ring + slot * kStage, vtile = ktile + kTile;
-          float sc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+        }
+        float sc[kPage];
 #pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            uint32_t a[4], bq[4];
-            ldmatrix_x4(a, qbase + kk * 32);
-            ldmatrix_x4(bq, swz(ktile, kt_t, 2 * kk + kt_c));
-            mma_bf16_16x8x16(sc[0], a, bq[0], bq[1]);
-            mma_bf16_16x8x16(sc[1], a, bq[2], bq[3]);
-          }
+        for (int t = 0; t < kPage; ++t) sc[t] = -INFINITY;
+        const uint32_t scol = kSPCol + sb * 64;
+        if (has && ok) {
+          uint32_t raw[16];
+          tmem_ld16(tl + scol + jp * kPage, raw);
+          tmem_ld_wait();
 #pragma unroll
-          for (int nt = 0; nt < 2; ++nt)
+          for (int t = 0; t < kPage; ++t) sc[t] = __uint_as_float(raw[t]);
+        }
+        // masks: token count of the page, and a suffix page is visible to one row only
+        const bool rowok = has && ok && rloc >= 0 && (sel < 0 || sel == rloc);
+        float mx = -INFINITY;
 #pragma unroll
-            for (int ee = 0; ee < 4; ++ee) {
-              const int t = nt * 8 + col + (ee & 1);
-              const bool ok = (t < tok) && (ee < 2 ? ok0 : ok1);
-              sc[nt][ee] = ok ? sc[nt][ee] * p.scale_log2 : -INFINITY;
+        for (int t = 0; t < kPage; ++t) {
+          const float v = (rowok && t < tok) ? sc[t] * p.scale_log2 : -INFINITY;
+          sc[t] = v;
+          mx = fmaxf(mx, v);
+        }
+        if (W > 1) {
+          // the group's row max over the quarter's page slots; the barrier also
+          // orders every warp's S reads before the P writes that overwrite them
+          float* rm = rmax + (gi & 1) * 4 * kRows;
+          rm[pj * kRows + tlane] = mx;
+          tc_fence_before();
+          soft_sync();
+          tc_fence_after();
+          mx = rm[tlane];
+          for (int w = 1; w < W; ++w) mx = fmaxf(mx, rm[w * kRows + tlane]);
+        }
+        const bool need = mx > m_used + kRescaleLog2;
+        if (__any_sync(0xffffffffu, need)) {
+          const float nm = need ? mx : m_used;
+          const float f = (m_used == -INFINITY) ? 0.f : exp2f(m_used - nm);
+          const int pg = gi - 1;
+          if (k0 > 0 && ok && !wwait(&p_empty[pg % kSPBufs], (uint32_t)(pg / kSPBufs) & 1u, abort_flag)) ok = false;
+          if (k0 > 0 && ok) {
+            // O holds this piece's earlier groups: the last PV is done; rescale this warp's columns
+            tc_fence_after();
+#pragma unroll 1
+            for (int cc = 0; cc < ocols; cc += 16) {
+              uint32_t raw[16];
+              const uint32_t col = kOCol + pj * ocols + cc;
+              tmem_ld16(tl + col, raw);
+              tmem_ld_wait();
+#pragma unroll
+              for (int t = 0; t < 16; ++t) raw[t] = __float_as_uint(__uint_as_float(raw[t]) * f);
+              tmem_st16(tl + col, raw);
             }
-          float mx0 = fmaxf(fmaxf(sc[0][0], sc[0][1]), fmaxf(sc[1][0], sc[1][1]));
-          float mx1 = fmaxf(fmaxf(sc[0][2], sc[0][3]), fmaxf(sc[1][2], sc[1][3]));
-          mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-          mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-          mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-          mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-          const float n0 = fmaxf(m0, mx0), n1 = fmaxf(m1, mx1);
-          if (__any_sync(0xffffffffu, n0 != m0 || n1 != m1)) {
-            // the running max moved for some row of the tile: rescale
-            const float al0 = (n0 == m0) ? 1.f : exp2f(m0 - n0);
-            const float al1 = (n1 == m1) ? 1.f : exp2f(m1 - n1);
-            l0 *= al0;
-            l1 *= al1;
-#pragma unroll
-            for (int i = 0; i < D / 8; ++i) {
-              o[i][0] *= al0;
-              o[i][1] *= al0;
-              o[i][2] *= al1;
-              o[i][3] *= al1;
-            }
-            m0 = n0;
-            m1 = n1;
+            tmem_st_wait();
           }
-          const float r0 = (m0 == -INFINITY) ? 0.f : m0, r1 = (m1 == -INFINITY) ? 0.f : m1;
-          float pr[2][4];
-#pragma unroll
-          for (int nt = 0; nt < 2; ++nt) {
-            pr[nt][0] = exp2f(sc[nt][0] - r0);
-            pr[nt][1] = exp2f(sc[nt][1] - r0);
-            pr[nt][2] = exp2f(sc[nt][2] - r1);
-            pr[nt][3] = exp2f(sc[nt][3] - r1);
-          }
-          l0 += (pr[0][0] + pr[0][1]) + (pr[1][0] + pr[1][1]);
-          l1 += (pr[0][2] + pr[0][3]) + (pr[1][2] + pr[1][3]);
-          uint32_t pa[4];
-          pa[0] = pack_bf16x2(pr[0][0], pr[0][1]);
-          pa[1] = pack_bf16x2(pr[0][2], pr[0][3]);
-          pa[2] = pack_bf16x2(pr[1][0], pr[1][1]);
-          pa[3] = pack_bf16x2(pr[1][2], pr[1][3]);
-#pragma unroll
-          for (int np = 0; np < D / 16; ++np) {
-            uint32_t bv[4];
-            ldmatrix_x4_trans(bv, swz(vtile, vt_t, 2 * np + vt_c));
-            mma_bf16_16x8x16(o[2 * np], pa, bv[0], bv[1]);
-            mma_bf16_16x8x16(o[2 * np + 1], pa, bv[2], bv[3]);
-          }
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&empty_bar[slot]);
-          slot += TS;
-          if (slot >= nst) {
-            slot -= nst;
-            phase ^= 1u;
-          }
+          l *= f;
+          m_used = nm;
         }
-        l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
-        l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
-        l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
-        l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-        if ((lane & 3) == 0) {
-          mls[(ts * n_mt + mt) * 16 + (lane >> 2)] = make_float2(m0, l0);
-          mls[(ts * n_mt + mt) * 16 + (lane >> 2) + 8] = make_float2(m1, l1);
+        const float ref = (m_used == -INFINITY) ? 0.f : m_used;
+        uint32_t pk[kPage / 2];
+#pragma unroll
+        for (int t = 0; t < kPage; t += 2) {
+          const float p0 = sc[t] == -INFINITY ? 0.f : exp2f(sc[t] - ref);
+          const float p1 = sc[t + 1] == -INFINITY ? 0.f : exp2f(sc[t + 1] - ref);
+          l += p0 + p1;
+          pk[t / 2] = pack_bf16x2(p0, p1);
         }
+        if (has && ok) tmem_st8(tl + scol + jp * 8, pk);  // P of this page, over its S columns
+        if (R > 1 && pj == 0 && ok) {
+          // the other copies' pages contribute nothing to this copy's O
+          const uint32_t zero[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+#pragma unroll
+          for (int jj = 0; jj < kGroupPages; ++jj)
+            if (jj < ng && jj % R != cp) tmem_st8(tl + scol + jj * 8, zero);
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_full[sb]);
+        ++gi;
       }
-      consumer_sync();
-      // ---- combine the token slices: O = sum_t 2^(m_t - M) O_t --------------
-      if (busy) {
-        float M0 = -INFINITY, M1 = -INFINITY;
-        for (int t = 0; t < TS; ++t) {
-          M0 = fmaxf(M0, mls[(t * n_mt + mt) * 16 + (lane >> 2)].x);
-          M1 = fmaxf(M1, mls[(t * n_mt + mt) * 16 + (lane >> 2) + 8].x);
-        }
-        const float f0 = (m0 == -INFINITY) ? 0.f : exp2f(m0 - M0);
-        const float f1 = (m1 == -INFINITY) ? 0.f : exp2f(m1 - M1);
-        float* a0 = acc + (mt * 16 + (lane >> 2)) * kAccStride + col;
-        float* a1 = a0 + 8 * kAccStride;
-        if (f0 != 0.f) {
-#pragma unroll
-          for (int i = 0; i < D / 8; ++i) {
-            atomicAdd(a0 + i * 8, f0 * o[i][0]);
-            atomicAdd(a0 + i * 8 + 1, f0 * o[i][1]);
-          }
-        }
-        if (f1 != 0.f) {
-#pragma unroll
-          for (int i = 0; i < D / 8; ++i) {
-            atomicAdd(a1 + i * 8, f1 * o[i][2]);
-            atomicAdd(a1 + i * 8 + 1, f1 * o[i][3]);
-          }
-        }
+      // ---- end of the piece: O is final once the last group's PV completes ----
+      const int lg = gi - 1;
+      if (ok && !wwait(&p_empty[lg % kSPBufs], (uint32_t)(lg / kSPBufs) & 1u, abort_flag)) ok = false;
+      tc_fence_after();
+      // the quarter's row sum over its W warps
+      float Lq = l;
+      if (W > 1) {
+        rsum[pj * kRows + tlane] = l;
+        soft_sync();
+        Lq = rsum[tlane];
+        for (int w = 1; w < W; ++w) Lq += rsum[w * kRows + tlane];
       }
-      // one thread snapshots the abort flag (the producer may set it at any time)
-      // so that every consumer takes the same branch below
-      if (tid == 0) s_piece_abort = *(volatile int32_t*)&s_abort;
-      consumer_sync();
-      const bool aborted = s_piece_abort != 0;
+      // the copies' (m, l) -> the piece's max M and sum L; copy c's O is weighted by 2^(m_c - M)
+      float M = m_used, Ls = Lq, wself = 1.f;
+      if (R > 1) {
+        if (pj == 0) mlx[tlane] = make_float2(m_used, Lq);
+        soft_sync();
+        M = -INFINITY;
+        for (int c2 = 0; c2 < R; ++c2) M = fmaxf(M, mlx[(c2 * qpc + rb) * 32 + lane].x);
+        Ls = 0.f;
+        for (int c2 = 0; c2 < R; ++c2) {
+          const float2 ml = mlx[(c2 * qpc + rb) * 32 + lane];
+          if (ml.x != -INFINITY) Ls += exp2f(ml.x - M) * ml.y;
+        }
+        wself = (m_used == -INFINITY) ? 0.f : exp2f(m_used - M);
+      }
       const int first = cta_of(cur.start, T, Ceff), last = cta_of(cur.start + cur.n - 1, T, Ceff);
-      // (M, L) of query i of this piece from the token-slice states
-      auto piece_ml = [&](int i) {
-        const int pm = i >> 4, pr = i & 15;
-        float M = -INFINITY;
-        for (int t = 0; t < TS; ++t) M = fmaxf(M, mls[(t * n_mt + pm) * 16 + pr].x);
-        float Ls = 0.f;
-        if (M != -INFINITY)
-          for (int t = 0; t < TS; ++t) {
-            const float2 v = mls[(t * n_mt + pm) * 16 + pr];
-            Ls += v.y * exp2f(v.x - M);
-          }
-        return make_float2(M, Ls);
-      };
-      if (!aborted && first == last) {
-        // the whole job is in this CTA: normalise and write the output
-        for (int idx = tid; idx < nq * (D / 2); idx += kCThreads) {
-          const int i = idx / (D / 2), d = 2 * (idx % (D / 2));
-          const int r = cur.g * p.rpg + i / gq, hq = cur.h * gq + i % gq;
-          if (!row_on(p, r)) continue;
-          const float2 ml = piece_ml(i);
-          const float inv = ml.y > 0.f ? 1.f / ml.y : 0.f;
-          const float* a = acc + i * kAccStride + d;
-          *reinterpret_cast<uint32_t*>(p.out + ((int64_t)r * p.Hq + hq) * D + d) =
-              pack_bf16x2(a[0] * inv, a[1] * inv);
-          if (d == 0 && p.lse)
-            p.lse[(int64_t)r * p.Hq + hq] = ml.y > 0.f ? (ml.x + log2f(ml.y)) * kLn2 : -INFINITY;
-        }
-      } else if (!aborted) {
-        // partial of a split job -> slot (cta + job); the last piece merges
-        const int64_t s = (int64_t)c + j;
-        for (int idx = tid; idx < nq * (D / 4); idx += kCThreads) {
-          const int i = idx / (D / 4), d = 4 * (idx % (D / 4));
-          const float* a = acc + i * kAccStride + d;
-          *reinterpret_cast<float4*>(p.slot_o + (s * nq + i) * D + d) = make_float4(a[0], a[1], a[2], a[3]);
-          if (d == 0) p.slot_ml[s * nq + i] = piece_ml(i);
-        }
-        __threadfence();
-        consumer_sync();
-        if (tid == 0) {
-          const int prev = atomicAdd(p.ticket + j, 1);
-          s_last = (prev == last - first);
-          if (s_last) __threadfence();
-        }
-        consumer_sync();
-        if (s_last) {
-          constexpr int kPer = D / 32;
-          for (int i = warp; i < nq; i += kCWarps) {
-            const int r = cur.g * p.rpg + i / gq, hq = cur.h * gq + i % gq;
-            if (!row_on(p, r)) continue;
-            float M = -INFINITY;
-            for (int cc = first; cc <= last; ++cc)
-              M = fmaxf(M, __ldcg(&p.slot_ml[((int64_t)cc + j) * nq + i].x));
-            float accv[kPer];
+      const bool mine_row = r < nq && cp == 0;
+      const int rr = r < nq ? cur.g * p.rpg + r / gq : 0, hq = r < nq ? cur.h * gq + r % gq : 0;
+      const bool write_row = mine_row && row_on(p, rr);
+      const int64_t s_idx = (int64_t)c + j;
+      const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+      // after an abort the piece's outputs are not written (the status word says so)
+      const bool out_ok = __all_sync(0xffffffffu, ok && !*abort_flag);
+      // O, 16 columns per round; copies >= 1 pass theirs to copy 0 through shared
+      // memory (double-buffered, so one barrier per round)
+      const int my_stage = ((cp - 1) * qpc + rb) * W + pj;  // (for copies >= 1)
+      const int stage_n = (R - 1) * qpc * W;  // staging rows of 32 lanes x 16 floats per buffer
+#pragma unroll 1
+      for (int cc = 0; cc < ocols; cc += 16) {
+        const int col = pj * ocols + cc;
+        float o[16];
+        if (out_ok) {
+          uint32_t raw[16];
+          tmem_ld16(tl + kOCol + col, raw);
+          tmem_ld_wait();
 #pragma unroll
-            for (int t = 0; t < kPer; ++t) accv[t] = 0.f;
-            float Ls = 0.f;
-            if (M != -INFINITY) {
-              for (int cc = first; cc <= last; ++cc) {
-                const int64_t si = ((int64_t)cc + j) * nq + i;
-                const float2 ml = __ldcg(&p.slot_ml[si]);
-                if (ml.y == 0.f) continue;
-                const float w = exp2f(ml.x - M);
-                Ls += w * ml.y;
-                const float* po = p.slot_o + si * D + lane * kPer;
-                if constexpr (kPer == 4) {
-                  const float4 v = __ldcg(reinterpret_cast<const float4*>(po));
-                  accv[0] += w * v.x;
-                  accv[1] += w * v.y;
-                  accv[2] += w * v.z;
-                  accv[3] += w * v.w;
-                } else {
-                  const float2 v = __ldcg(reinterpret_cast<const float2*>(po));
-                  accv[0] += w * v.x;
-                  accv[1] += w * v.y;
-                }
+          for (int t = 0; t < 16; ++t) o[t] = __uint_as_float(raw[t]) * wself;
+        }
+        if (R > 1) {
+          float4* sb4 = stage + ((cc / 16) & 1) * (stage_n * 4 * 32);
+          if (cp > 0 && out_ok) {
+#pragma unroll
+            for (int t = 0; t < 4; ++t)
+              sb4[(my_stage * 4 + t) * 32 + lane] = make_float4(o[4 * t], o[4 * t + 1], o[4 * t + 2], o[4 * t + 3]);
+          }
+          soft_sync();
+          if (cp == 0 && out_ok) {
+#pragma unroll 1
+            for (int c2 = 1; c2 < R; ++c2) {
+              const float4* src4 = sb4 + ((((c2 - 1) * qpc + rb) * W + pj) * 4) * 32 + lane;
+#pragma unroll
+              for (int t = 0; t < 4; ++t) {
+                const float4 v = src4[t * 32];
+                o[4 * t] += v.x;
+                o[4 * t + 1] += v.y;
+                o[4 * t + 2] += v.z;
+                o[4 * t + 3] += v.w;
               }
             }
-            const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-            __nv_bfloat16* dst = p.out + ((int64_t)r * p.Hq + hq) * D + lane * kPer;
-            if constexpr (kPer == 4) {
-              uint2 pk;
-              pk.x = pack_bf16x2(accv[0] * inv, accv[1] * inv);
-              pk.y = pack_bf16x2(accv[2] * inv, accv[3] * inv);
-              *reinterpret_cast<uint2*>(dst) = pk;
-            } else {
-              *reinterpret_cast<uint32_t*>(dst) = pack_bf16x2(accv[0] * inv, accv[1] * inv);
-            }
-            if (p.lse && lane == 0)
-              p.lse[(int64_t)r * p.Hq + hq] = Ls > 0.f ? (M + log2f(Ls)) * kLn2 : -INFINITY;
           }
-          if (tid == 0) p.ticket[j] = 0;
+        }
+        if (!out_ok) continue;
+        if (first == last) {
+          if (write_row) {
+            uint4* dst = reinterpret_cast<uint4*>(p.out + ((int64_t)rr * p.Hq + hq) * D + col);
+            dst[0] = make_uint4(pack_bf16x2(o[0] * inv, o[1] * inv), pack_bf16x2(o[2] * inv, o[3] * inv),
+                                pack_bf16x2(o[4] * inv, o[5] * inv), pack_bf16x2(o[6] * inv, o[7] * inv));
+            dst[1] = make_uint4(pack_bf16x2(o[8] * inv, o[9] * inv), pack_bf16x2(o[10] * inv, o[11] * inv),
+                                pack_bf16x2(o[12] * inv, o[13] * inv), pack_bf16x2(o[14] * inv, o[15] * inv));
+          }
+        } else if (mine_row) {
+          float4* dst = reinterpret_cast<float4*>(p.slot_o + (s_idx * nq + r) * D + col);
+#pragma unroll
+          for (int t = 0; t < 4; ++t) dst[t] = make_float4(o[4 * t], o[4 * t + 1], o[4 * t + 2], o[4 * t + 3]);
         }
       }
-      consumer_sync();  // Q, acc and the slice states are reused by the next piece
-      x0 = pe;
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&o_free);
+      if (first == last) {
+        if (out_ok && pj == 0 && write_row && p.lse)
+          p.lse[(int64_t)rr * p.Hq + hq] = Ls > 0.f ? (M + log2f(Ls)) * kLn2 : -INFINITY;
+      } else if (out_ok && pj == 0 && mine_row) {
+        p.slot_ml[s_idx * nq + r] = make_float2(M, Ls);  // the merge kernel finishes the job
+      }
+      soft_sync();  // the exchange buffers are reused at the next piece
+      ++pc;
+      x0 += n_in;
       if (x0 < e) cur = next_job(p, gpre, cur);
     }
   }
+  tc_fence_before();
   __syncthreads();
-  if (s_abort && tid == 0) {
-    // a copy did not land: report, and wait (bounded) for the copies still in flight
-    flag(p.dev_status, RGD_DEV_WAIT_TIMEOUT);
-    for (int li = max(0, s_issued - nst); li < s_issued; ++li) mbar_wait(&full_bar[li % nst], (li / nst) & 1);
+  if (*abort_flag) {
+    // a wait gave up: report, and let copies and MMAs still in flight drain (bounded)
+    if (tid == 0) {
+      flag(p.dev_status, RGD_DEV_WAIT_TIMEOUT);
+      const int issued = s_issued;
+      for (int g = max(0, issued - ns); g < issued; ++g) mbar_wait(&full_bar[g % ns], (g / ns) & 1);
+    }
+    if (warp == kMmaWarp && lane == 0) {
+      umma_commit(&mma_done);  // arrives once every MMA this thread issued has completed
+      mbar_wait(&mma_done, 0);
+    }
+    __syncthreads();
+  }
+  tc_fence_after();
+  if (warp == kMmaWarp) tmem_dealloc(tmem, kTmemCols);
+}
+
+// Merge of a split job's partials (one block per job): with piece c holding the
+// unnormalised o_c and (m_c, l_c) in log2 units,
+//   out = sum_c 2^(m_c - M) o_c / sum_c 2^(m_c - M) l_c,  M = max_c m_c,
+//   lse = ln 2 * (M + log2 sum_c 2^(m_c - M) l_c).
+// Jobs held by one block were finished by the attention kernel.
+constexpr int kMergeThreads = 256;
+
+template <int D>
+__global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnParams p) {
+  const int j = blockIdx.x;
+  const int g = j / p.Hkv, h = j % p.Hkv;
+  const int32_t* gp = p.gpre_ws;
+  const int64_t T = (int64_t)p.Hkv * gp[p.G];
+  const int n = gp[g + 1] - gp[g];
+  if (n == 0) return;
+  const int Ceff = (int)min((int64_t)p.C, T);
+  const int64_t start = (int64_t)p.Hkv * gp[g] + (int64_t)h * n;
+  const int first = cta_of(start, T, Ceff), last = cta_of(start + n - 1, T, Ceff);
+  if (first == last) return;
+  const int nq = p.nq, gq = p.gq;
+  constexpr int kChunks = D / 4;
+  for (int item = threadIdx.x; item < nq * kChunks; item += kMergeThreads) {
+    const int i = item / kChunks, c4 = item % kChunks;
+    const int r = g * p.rpg + i / gq, hq = h * gq + i % gq;
+    if (!row_on(p, r)) continue;
+    float M = -INFINITY;
+    for (int cc = first; cc <= last; ++cc) M = fmaxf(M, p.slot_ml[((int64_t)cc + j) * nq + i].x);
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    float Ls = 0.f;
+    if (M != -INFINITY) {
+      for (int cc = first; cc <= last; ++cc) {
+        const int64_t si = ((int64_t)cc + j) * nq + i;
+        const float2 ml = p.slot_ml[si];
+        if (ml.y == 0.f) continue;
+        const float w = exp2f(ml.x - M);
+        Ls += w * ml.y;
+        const float4 v = reinterpret_cast<const float4*>(p.slot_o + si * D)[c4];
+        acc.x += w * v.x;
+        acc.y += w * v.y;
+        acc.z += w * v.z;
+        acc.w += w * v.w;
+      }
+    }
+    const float iv = Ls > 0.f ? 1.f / Ls : 0.f;
+    uint2 pk;
+    pk.x = pack_bf16x2(acc.x * iv, acc.y * iv);
+    pk.y = pack_bf16x2(acc.z * iv, acc.w * iv);
+    reinterpret_cast<uint2*>(p.out + ((int64_t)r * p.Hq + hq) * D)[c4] = pk;
+    if (p.lse && c4 == 0) p.lse[(int64_t)r * p.Hq + hq] = Ls > 0.f ? (M + log2f(Ls)) * kLn2 : -INFINITY;
   }
 }
 
@@ -601,15 +859,15 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
   return fn;
 }
 
-int make_kv_map(CUtensorMap* map, const void* base, int64_t rows, int D) {
+int make_kv_map(CUtensorMap* map, const void* base, int64_t rows, int D, int box_halves) {
   auto fn = get_encode_fn();
   if (!fn) return set_error(RGD_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
   // View each 16-token page-head tile as (64 columns) x (16 rows) x (D/64 halves):
-  // one box is the whole tile, laid out in shared memory half-major with the
-  // 128-byte swizzle (16-byte chunk index XOR row index mod 8).
+  // a box is one half or the whole tile, laid out in shared memory half-major
+  // with the 128-byte swizzle (16-byte chunk index XOR row index mod 8).
   cuuint64_t dims[3] = {64, (cuuint64_t)rows, (cuuint64_t)(D / 64)};
   cuuint64_t strides[2] = {(cuuint64_t)D * 2, 128};
-  cuuint32_t box[3] = {64, (cuuint32_t)kPage, (cuuint32_t)(D / 64)};
+  cuuint32_t box[3] = {64, (cuuint32_t)kPage, (cuuint32_t)box_halves};
   cuuint32_t estr[3] = {1, 1, 1};
   CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -626,9 +884,9 @@ int device_sm_count() {
 }
 
 struct Plan {
-  int nq, n_mt, TS, nst, C, J;
+  int nq, nslots, C, J;
   SmemLayout smem;
-  size_t ticket_off, ml_off, o_off, total;
+  size_t gpre_off, ml_off, o_off, total;
 };
 
 int check_shape(const rgd_attn_shape* s) {
@@ -658,42 +916,32 @@ int check_shape(const rgd_attn_shape* s) {
 int make_plan(const rgd_attn_shape* s, Plan* pl) {
   if (int rc = check_shape(s)) return rc;
   pl->nq = s->rows_per_group * (s->num_q_heads / s->num_kv_heads);
-  pl->n_mt = (pl->nq + 15) / 16;
-  pl->TS = kCWarps / pl->n_mt;
   pl->C = s->num_ctas > 0 ? s->num_ctas : device_sm_count();
   if (pl->C <= 0) return set_error(RGD_ERR_CUDA, "could not query the device's SM count");
   pl->J = s->num_groups * s->num_kv_heads;
-  pl->nst = (kMaxStages / pl->TS) * pl->TS;
+  // The ring holds at least three page groups: a group's slot is released by
+  // its PV, which is issued after the next group's QK.
+  pl->nslots = kMaxSlots;
   for (;;) {
-    pl->smem = s->head_dim == 128 ? smem_layout<128>(pl->nst, pl->n_mt, pl->TS, s->num_groups)
-                                  : smem_layout<64>(pl->nst, pl->n_mt, pl->TS, s->num_groups);
+    pl->smem = s->head_dim == 128 ? smem_layout<128>(pl->nslots, s->num_groups) : smem_layout<64>(pl->nslots, s->num_groups);
     if (pl->smem.total <= kSmemLimit) break;
-    if (pl->nst <= pl->TS)
+    if (pl->nslots <= 3)
       return set_error(RGD_ERR_UNSUPPORTED, "shape needs more shared memory than an SM has (too many groups?)");
-    pl->nst -= pl->TS;
+    --pl->nslots;
   }
   auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
-  const size_t nslots = (size_t)pl->C + pl->J - 1;
-  pl->ticket_off = 0;
-  pl->ml_off = up((size_t)pl->J * sizeof(int32_t));
-  pl->o_off = pl->ml_off + up(nslots * pl->nq * sizeof(float2));
-  pl->total = pl->o_off + up(nslots * pl->nq * s->head_dim * sizeof(float));
+  const size_t n_part = (size_t)pl->C + pl->J - 1;  // partial-result slots
+  pl->gpre_off = 0;
+  pl->ml_off = up((size_t)(s->num_groups + 1) * sizeof(int32_t));
+  pl->o_off = pl->ml_off + up(n_part * pl->nq * sizeof(float2));
+  pl->total = pl->o_off + up(n_part * pl->nq * s->head_dim * sizeof(float));
   return RGD_OK;
 }
 
 // Workspace fields used by the allocation-free entry point below.
-struct WsLayout {
-  size_t ml_off, total;
-};
-
-WsLayout ws_layout(const rgd_attn_shape* s) {
+size_t ws_total(const rgd_attn_shape* s) {
   Plan pl;
-  WsLayout w{0, 0};
-  if (make_plan(s, &pl) == RGD_OK) {
-    w.ml_off = pl.ml_off;
-    w.total = pl.total;
-  }
-  return w;
+  return make_plan(s, &pl) == RGD_OK ? pl.total : 0;
 }
 
 }  // namespace
@@ -729,8 +977,8 @@ extern "C" int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf1
 
   CUtensorMap tmK, tmV;
   const int64_t kv_rows = (int64_t)s.num_pages * s.num_kv_heads * kPage;
-  if (int rc = make_kv_map(&tmK, k_pages, kv_rows, s.head_dim)) return rc;
-  if (int rc = make_kv_map(&tmV, v_pages, kv_rows, s.head_dim)) return rc;
+  if (int rc = make_kv_map(&tmK, k_pages, kv_rows, s.head_dim, 1)) return rc;                // one half per box
+  if (int rc = make_kv_map(&tmV, v_pages, kv_rows, s.head_dim, s.head_dim / 64)) return rc;  // whole tile
 
   AttnParams p;
   p.q = reinterpret_cast<const __nv_bfloat16*>(q);
@@ -742,7 +990,7 @@ extern "C" int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf1
   p.out = reinterpret_cast<__nv_bfloat16*>(out);
   p.lse = lse;
   uint8_t* ws = static_cast<uint8_t*>(workspace);
-  p.ticket = reinterpret_cast<int32_t*>(ws + pl.ticket_off);
+  p.gpre_ws = reinterpret_cast<int32_t*>(ws + pl.gpre_off);
   p.slot_ml = reinterpret_cast<float2*>(ws + pl.ml_off);
   p.slot_o = reinterpret_cast<float*>(ws + pl.o_off);
   p.dev_status = dev_status;
@@ -755,21 +1003,21 @@ extern "C" int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf1
   p.max_pp = s.max_prompt_pages;
   p.max_sp = s.max_suffix_pages;
   p.nq = pl.nq;
-  p.n_mt = pl.n_mt;
-  p.TS = pl.TS;
-  p.nst = pl.nst;
+  p.nslots = pl.nslots;
   p.C = pl.C;
   p.scale_log2 = softmax_scale * kLog2e;
 
   cudaStream_t st = (cudaStream_t)stream;
   if (s.head_dim == 128) {
     static bool done = false;
-    if (int rc = ensure_smem(attn_persistent_kernel<128>, kSmemLimit, &done)) return rc;
-    attn_persistent_kernel<128><<<pl.C, kAttnThreads, pl.smem.total, st>>>(tmK, tmV, p);
+    if (int rc = ensure_smem(attn_tc_kernel<128>, kSmemLimit, &done)) return rc;
+    attn_tc_kernel<128><<<pl.C, kAttnThreads, pl.smem.total, st>>>(tmK, tmV, p);
+    attn_merge_kernel<128><<<pl.J, kMergeThreads, 0, st>>>(p);
   } else {
     static bool done = false;
-    if (int rc = ensure_smem(attn_persistent_kernel<64>, kSmemLimit, &done)) return rc;
-    attn_persistent_kernel<64><<<pl.C, kAttnThreads, pl.smem.total, st>>>(tmK, tmV, p);
+    if (int rc = ensure_smem(attn_tc_kernel<64>, kSmemLimit, &done)) return rc;
+    attn_tc_kernel<64><<<pl.C, kAttnThreads, pl.smem.total, st>>>(tmK, tmV, p);
+    attn_merge_kernel<64><<<pl.J, kMergeThreads, 0, st>>>(p);
   }
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? RGD_OK : cuda_error(e, "attention launch");
@@ -778,7 +1026,7 @@ extern "C" int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf1
 // ---------------------------------------------------------------------------
 // Allocation-free variant of rgd_prefix_decode_attn
 // ---------------------------------------------------------------------------
-// The split partials and tickets live in a fixed file-scope device array
+// The split partials live in a fixed file-scope device array
 // instead of a caller-provided workspace.  The array exists once per device in
 // every process that loads the library, for the life of the process.
 namespace rgd {
@@ -802,12 +1050,12 @@ extern "C" int rgd_prefix_decode_attn_noalloc(const rgd_attn_shape* shape, const
                                               float* lse, int32_t* dev_status, rgd_stream_t stream) {
   clear_error();
   if (int rc = check_shape(shape)) return rc;
-  const WsLayout w = ws_layout(shape);
-  if (w.total > kStaticScratchBytes)
+  const size_t need = ws_total(shape);
+  if (need > kStaticScratchBytes)
     return set_error(RGD_ERR_UNSUPPORTED,
                      "rgd_prefix_decode_attn_noalloc: this shape needs %zu bytes of scratch; the static "
                      "scratch holds %zu (use rgd_prefix_decode_attn with a workspace)",
-                     w.total, kStaticScratchBytes);
+                     need, kStaticScratchBytes);
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
@@ -825,9 +1073,8 @@ extern "C" int rgd_prefix_decode_attn_noalloc(const rgd_attn_shape* shape, const
     }
     scratch = g_scratch_ptr[dev];
   }
-  // the array keeps the previous call's contents: the tickets must start at zero
-  e = cudaMemsetAsync(scratch, 0, w.ml_off, (cudaStream_t)stream);
-  if (e != cudaSuccess) return cuda_error(e, "cudaMemsetAsync(scratch tickets)");
+  // the array keeps the previous call's contents; every value a call reads from
+  // it was written earlier in the same call, so nothing needs clearing
   return rgd_prefix_decode_attn(shape, q, k_pages, v_pages, prompt_block_table, prompt_len, suffix_block_table,
                                 suffix_len, row_active, softmax_scale, out, lse, scratch, kStaticScratchBytes,
                                 dev_status, stream);

@@ -2,7 +2,7 @@
 
 Moves a :class:`workloads.AttnCase` / :class:`workloads.HeadCase` to the GPU as
 torch tensors laid out the way the C ABI expects, and allocates the outputs and
-the zero-filled attention workspace.  No arithmetic of the method happens here.
+the attention workspace.  No arithmetic of the method happens here.
 """
 from __future__ import annotations
 

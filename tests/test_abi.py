@@ -54,7 +54,7 @@ def test_workspace_size_grows_with_blocks(lib_path):
     a = lib.rgd_prefix_decode_attn_workspace_size(ctypes.byref(s))
     s.num_ctas = 400
     b = lib.rgd_prefix_decode_attn_workspace_size(ctypes.byref(s))
-    # tickets for 128 jobs + (ctas + jobs - 1) partial slots of 20 queries x (128 + 2) floats
+    # the page-count prefix of 16 groups + (ctas + jobs - 1) partial slots of 20 queries x (128 + 2) floats
     grow = 300 * 20 * 128 * 4 + 300 * 20 * 8
     assert grow <= b - a < grow + 512  # each region is padded to 256 bytes
     s.reserved = 1

@@ -39,7 +39,7 @@ def _both(case):
 
 def test_noalloc_matches_workspace_entry_point_twice(gpu_lib):
     # first call: the Llama-3-8B-shaped step; second call: a smaller shape with
-    # masked rows, which must not see the first call's tickets or partials
+    # masked rows, which must not see the first call's partials
     _both(workloads.llama8b(seed=2).attn)
     active = np.array([1, 0, 1, 1, 1, 1, 0, 0, 1], np.uint8)
     _both(workloads.make_attn_case("second", 3, 3, 8, 2, 64, [0, 37, 300], [0, 1, 16, 17, 40, 0, 5, 33, 64],
