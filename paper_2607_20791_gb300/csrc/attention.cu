@@ -17,7 +17,7 @@
 // like the jobs -- and a second, small kernel merges each split job's partials
 // by log-sum-exp (Sec. 3's shared-prefix split is the same identity).
 //
-// Inside a block (576 threads) the tensor memory holds Q, S / P and O, so the
+// Inside a block (608 threads) the tensor memory holds Q, S / P and O, so the
 // tensor cores read only K and V from shared memory -- the bytes that come from
 // HBM:
 //   * warp 16 (producer) streams the pages, four to a group, into a ring of
@@ -27,21 +27,23 @@
 //     its N, so the number of MMAs, not their size, is what counts), each V
 //     tile as one box; every lane issues its own page, since one issuing
 //     thread is copy-rate bound;
-//   * warp 17 allocates the tensor memory and its lane 0 issues every MMA: for a
-//     group of up to 4 pages, S = Q K^T (A = Q from TMEM, M = 128 query rows,
-//     N = 16 x pages) into one of three S/P buffers, and, once the
-//     softmax warps have turned S into bf16 P in place, O += P V per page (A = P
-//     from TMEM, N = the head dimension, V read MN-major from its tile); one
-//     commit after the group's PV hands its slot back to the producer;
-//   * warps 0-15: warp w owns TMEM lanes 32(w%4)..+31 (query rows) and page w/4
-//     of the group, so every thread handles the 16 scores of one row and one
-//     page: the masks, the group's row max (exchanged through shared memory),
-//     the online softmax in fp32 (the running max is only moved, and O rescaled
-//     in TMEM, when a row's max grows by more than 2^8) and its 16 bf16 P values;
-//     they also write Q into TMEM, and at the end of a job piece the four warps
-//     of a lane quarter each read a quarter of O's columns and write the output
-//     or the partial.  Warps whose lane quarter holds only padding rows (>= the
-//     job's query count) sit out.
+//   * warp 17 allocates the tensor memory and its lane 0 issues, for a group
+//     of up to 4 pages, S = Q K^T (A = Q from TMEM, M = 128 query rows,
+//     N = 16 x pages) into one of three S/P buffers; once the softmax warps
+//     have turned S into bf16 P in place, lane 0 of warp 18 issues O += P V per
+//     page (A = P from TMEM, N = the head dimension, V read MN-major from its
+//     tile), and one commit after the group's PV hands its slot back to the
+//     producer;
+//   * warps 0-15 (softmax): warp w can reach TMEM lanes 32(w%4)..+31 only.  The
+//     job's queries are held in as many copies as fit in the 128 lanes; a
+//     softmax warp handles the 16 scores of one page for 32 query rows of one
+//     copy: the masks, the row max (shared through shared memory by the warps of
+//     a copy that share rows), the online softmax in fp32 (the running max is
+//     only moved, and O rescaled in TMEM, when a row's max grows by more than
+//     2^8) and its 16 bf16 P values.  They also write Q into TMEM, and at the end
+//     of a job piece every warp of a used lane quarter reads a quarter of O's
+//     columns; the copies are merged by log-sum-exp and the output or the
+//     partial written.
 // Every wait on an mbarrier is bounded; a timeout is reported in the status
 // word and every role stops.
 #include <cudaTypedefs.h>
@@ -59,8 +61,9 @@ constexpr int kPage = 16;
 constexpr int kSoftWarps = 16;                // warps 0-15: softmax / epilogue
 constexpr int kSoftThreads = kSoftWarps * 32;
 constexpr int kProducerWarp = 16;
-constexpr int kMmaWarp = 17;
-constexpr int kAttnThreads = 18 * 32;
+constexpr int kMmaWarp = 17;                  // QK issue (and the TMEM allocation)
+constexpr int kPvWarp = 18;                   // PV issue
+constexpr int kAttnThreads = 19 * 32;
 constexpr int kGroupPages = 4;                // pages per S / P buffer (64 tokens)
 constexpr int kMaxSlots = 8;                  // ring slots, one page group each
 constexpr int kSPBufs = 3;                    // S / P buffers in TMEM
@@ -119,8 +122,8 @@ __host__ __device__ inline SmemLayout smem_layout(int nslots, int G) {
   SmemLayout L;
   L.ring = 0;
   L.red = nslots * slot_bytes<D>();
-  // row-max exchange (2 buffers), row-sum exchange, per-lane (m, l), O staging (2 buffers)
-  L.gpre = L.red + (3 * 4 * kRows + 2 * kRows + 2 * 4 * 32 * 16) * 4;
+  // row-max exchange (2 buffers), row-sum exchange, per-lane running max, O staging
+  L.gpre = L.red + (3 * 4 * kRows + kRows + 12 * 4 * 32 * 4) * 4;
   L.gact = align_up(L.gpre + (G + 1) * 4, 16);
   L.desc = align_up(L.gact + G * 4, 16);
   L.total = align_up(L.desc + nslots * kGroupPages * 4, 16) + 1024;  // + slack for the 1024-byte aligned base
@@ -208,7 +211,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   int32_t* gpre = reinterpret_cast<int32_t*>(smem + L.gpre);
   uint32_t* descs = reinterpret_cast<uint32_t*>(smem + L.desc);
   __shared__ uint64_t full_bar[kMaxSlots], empty_bar[kMaxSlots];
-  __shared__ uint64_t s_full[kSPBufs], p_full[kSPBufs], p_empty[kSPBufs], q_full[2], q_empty[2], o_free, mma_done;
+  __shared__ uint64_t s_full[kSPBufs], p_full[kSPBufs], p_empty[kSPBufs], q_full[2], q_empty[2], o_free, mma_done[2];
   __shared__ int32_t s_abort, s_issued, s_wsum[kAttnThreads / 32];
   __shared__ uint32_t s_tmem;
   volatile int32_t* abort_flag = &s_abort;
@@ -222,7 +225,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int qpc = (p.nq + 31) / 32;         // lane quarters one copy of the queries spans
   const int R = 4 / qpc;                    // copies of the queries in the 128 lanes
   const int W = kGroupPages / R;            // softmax warps per quarter (pages per copy and group)
-  const int n_act = R * qpc * W;            // active softmax warps
+  const int n_soft = R * qpc * W;           // softmax warps of each group
+  const int n_piece = R * qpc * 4;          // warps that write Q and read O
 
   if (tid == 0) {
     for (int i = 0; i < ns; ++i) {
@@ -231,15 +235,16 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     }
     for (int i = 0; i < kSPBufs; ++i) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&p_full[i], n_act);
+      mbar_init(&p_full[i], n_soft);
       mbar_init(&p_empty[i], 1);
     }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&q_full[i], n_act);
+      mbar_init(&q_full[i], n_piece);
       mbar_init(&q_empty[i], 1);
     }
-    mbar_init(&o_free, n_act);
-    mbar_init(&mma_done, 1);
+    mbar_init(&o_free, n_piece);
+    mbar_init(&mma_done[0], 1);
+    mbar_init(&mma_done[1], 1);
     s_abort = 0;
     s_issued = 0;
     fence_mbar_init();
@@ -405,33 +410,17 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       }
     }
   } else if (warp == kMmaWarp) {
-    // ============================ MMA issue ===========================
+    // ============================ QK issue ============================
+    // One thread issues S = Q K^T for every group as soon as its pages have
+    // landed and its S / P buffer is free; the PV MMAs come from another warp,
+    // since an issuing thread spends ~60 cycles per MMA whatever its size (two
+    // issuers double the MMA rate; N = 64 MMAs take the tensor pipe ~32 cycles).
     // B descriptors are formed once; an MMA's B differs from the ring base only
     // in the start-address field (byte offset / 16).
     if (lane == 0 && b < e) {
       const uint64_t k_d = smem_desc(sbase, 1024, 1024, 2);
-      const uint64_t v_d = smem_desc(sbase, D == 128 ? kVLbo : 1024, D == 128 ? kVSbo : 1024, 2);
       int gi = 0, pc = 0;
-      // the previous group's PV waits until the next group's QK is issued
-      int pv_gi = -1, pv_n = 0, pv_first = 0, pv_pc = 0;
       bool ok = true;
-      auto issue_pv = [&]() {
-        const int pb = pv_gi % kSPBufs;
-        const int gs = pv_gi % ns;
-        if (!wait_or_abort(&p_full[pb], (uint32_t)(pv_gi / kSPBufs) & 1u, abort_flag)) return false;
-        if (pv_first && pv_pc >= 1 && !wait_or_abort(&o_free, (uint32_t)(pv_pc - 1) & 1u, abort_flag)) return false;
-        tc_fence_after();
-#pragma unroll
-        for (int j = 0; j < kGroupPages; ++j) {
-          if (j < pv_n)
-            umma_bf16_tmem_a(tmem + kOCol, tmem + kSPCol + pb * 64 + j * 8,
-                             v_d + (uint64_t)((gs * kSlot + kVOff + j * kTile) >> 4), kIdescPV,
-                             (pv_first && j == 0) ? 0u : 1u);
-        }
-        umma_commit(&p_empty[pb]);
-        umma_commit(&empty_bar[gs]);  // the slot's K and V are no longer read
-        return true;
-      };
       Job cur = job_at(p, gpre, b);
       int64_t x0 = b;
       while (ok && x0 < e) {
@@ -464,18 +453,50 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                              kk > 0 ? 1u : 0u);
           umma_commit(&s_full[sb]);
           if (k0 + ng == n_in) umma_commit(&q_empty[qb]);
-          if (pv_gi >= 0 && !issue_pv()) {
+          ++gi;
+        }
+        ++pc;
+        x0 += n_in;
+        if (x0 < e) cur = next_job(p, gpre, cur);
+      }
+    }
+  } else if (warp == kPvWarp) {
+    // ============================ PV issue ============================
+    // O += P V for every page of a group once the softmax has written its P
+    // (and, for a piece's first group, once the previous piece's O has been
+    // read); one commit then frees the S / P buffer, another the ring slot.
+    if (lane == 0 && b < e) {
+      const uint64_t v_d = smem_desc(sbase, D == 128 ? kVLbo : 1024, D == 128 ? kVSbo : 1024, 2);
+      int gi = 0, pc = 0;
+      bool ok = true;
+      Job cur = job_at(p, gpre, b);
+      int64_t x0 = b;
+      while (ok && x0 < e) {
+        const int n_in = (int)(min(e, cur.start + cur.n) - x0);
+        for (int k0 = 0; k0 < n_in; k0 += kGroupPages) {
+          const int ng = min(kGroupPages, n_in - k0);
+          const int pb = gi % kSPBufs;
+          const int gs = gi % ns;
+          if (!wait_or_abort(&p_full[pb], (uint32_t)(gi / kSPBufs) & 1u, abort_flag)) {
             ok = false;
             break;
           }
-          pv_gi = gi;
-          pv_n = ng;
-          pv_first = (k0 == 0);
-          pv_pc = pc;
+          if (k0 == 0 && pc >= 1 && !wait_or_abort(&o_free, (uint32_t)(pc - 1) & 1u, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+#pragma unroll
+          for (int j = 0; j < kGroupPages; ++j) {
+            if (j < ng)
+              umma_bf16_tmem_a(tmem + kOCol, tmem + kSPCol + pb * 64 + j * 8,
+                               v_d + (uint64_t)((gs * kSlot + kVOff + j * kTile) >> 4), kIdescPV,
+                               (k0 == 0 && j == 0) ? 0u : 1u);
+          }
+          umma_commit(&p_empty[pb]);
+          umma_commit(&empty_bar[gs]);  // the slot's K and V are no longer read
           ++gi;
         }
-        if (ok && pv_gi >= 0 && !issue_pv()) ok = false;
-        pv_gi = -1;
         ++pc;
         x0 += n_in;
         if (x0 < e) cur = next_job(p, gpre, cur);
@@ -489,30 +510,65 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     // with an online softmax of its own, and W = 4 / R warps of each of its
     // quarters (one page each) share that copy's running max; its P is zero in
     // the other copies' page columns, so O in its lanes sums its own pages only.
-    // The copies are merged by log-sum-exp at the end of the piece.  For nq <= 32
-    // each page of a group is thus handled on its own SM sub-partition (a warp
-    // can only reach its own lane quarter) and no warp waits for another between
-    // groups.
+    // For nq <= 32 each page of a group is thus handled on its own SM
+    // sub-partition (a warp can only reach its own lane quarter) and no warp
+    // waits for another between groups.  At the end of a job piece all four
+    // warps of every used quarter read O (a quarter of its columns each), and the
+    // copies are merged by log-sum-exp through shared memory; the next piece's Q
+    // is written before that, so its first QKs overlap the epilogue.
     const int nq = p.nq, gq = p.gq;
     const int qd = warp & 3, pj = warp >> 2;  // TMEM lane quarter; warp within the quarter
     const int cp = qd / qpc, rb = qd % qpc;   // copy; row block of the queries
-    const bool active = cp < R && pj < W;
+    const bool in_piece = cp < R;             // Q writes and the epilogue
+    const bool in_group = in_piece && pj < W; // the softmax of each group
     const int jp = cp + pj * R;               // this warp's page within a group
-    const int n_athr = n_act * 32;
-    auto soft_sync = [&]() { asm volatile("bar.sync 1, %0;" ::"r"(n_athr) : "memory"); };
+    auto soft_sync = [&]() { asm volatile("bar.sync 1, %0;" ::"r"(n_soft * 32) : "memory"); };
+    auto piece_sync = [&]() { asm volatile("bar.sync 2, %0;" ::"r"(n_piece * 32) : "memory"); };
     const int r = rb * 32 + lane;              // this thread's query
     const int rloc = r < nq ? r / gq : -2;     // its row within the group (suffix pages are per row)
     const int tlane = qd * 32 + lane;          // its TMEM lane
     const uint32_t tl = tmem + ((uint32_t)(qd * 32) << 16);
     float* rmax = reinterpret_cast<float*>(smem + L.red);  // [2][4][128] page-slot maxima
     float* rsum = rmax + 2 * 4 * kRows;                    // [4][128] page-slot row sums
-    float2* mlx = reinterpret_cast<float2*>(rsum + 4 * kRows);  // [128] (m, l) of each lane
-    float4* stage = reinterpret_cast<float4*>(mlx + kRows);     // [2][<= 4 * 32 * 4] O columns of copies >= 1
-    const int ocols = D / W;                   // O columns read / rescaled by each warp of a quarter
-    const int qcols = (D / 2) / W;             // Q columns (bf16 pairs) written by each warp of a quarter
+    float* mfin = rsum + 4 * kRows;                        // [128] running max at the piece end
+    float4* stage = reinterpret_cast<float4*>(mfin + kRows);  // [<= 12][4][32] O columns of copies >= 1
+    const int ocols = D / W;                   // O columns rescaled by each softmax warp of a quarter
+    constexpr int kEpiCols = D / 4;            // O columns read by each warp of a quarter at the end
+    constexpr int kQCols = D / 8;              // Q columns (bf16 pairs) written by each warp of a quarter
     // warp-uniform bounded wait (TMEM loads and stores that follow are warp-collective)
     auto wwait = [&](uint64_t* bar, uint32_t parity, volatile int32_t* flag) {
       return __all_sync(0xffffffffu, wait_or_abort(bar, parity, flag));
+    };
+    // this warp's share of its rows' queries for piece number `pn` of job `jb`
+    auto write_q = [&](const Job& jb, int pn) {
+      const int qb = pn & 1;
+      bool fine = true;
+      if (pn >= 2 && !wwait(&q_empty[qb], (uint32_t)((pn >> 1) - 1) & 1u, abort_flag)) fine = false;
+      if (fine) {
+        constexpr int kLd = kQCols / 4;  // uint4 loads: a column holds two bf16, a uint4 eight
+        uint4 qv[kLd];
+        if (r < nq) {
+          const int rr = jb.g * p.rpg + r / gq, hq = jb.h * gq + r % gq;
+          const uint4* src = reinterpret_cast<const uint4*>(p.q + ((int64_t)rr * p.Hq + hq) * D) + pj * kLd;
+#pragma unroll
+          for (int t = 0; t < kLd; ++t) qv[t] = __ldg(src + t);
+        } else {
+#pragma unroll
+          for (int t = 0; t < kLd; ++t) qv[t] = make_uint4(0u, 0u, 0u, 0u);
+        }
+        const uint32_t qcol = kQCol + qb * (D / 2) + pj * kQCols;
+#pragma unroll
+        for (int t = 0; t < kQCols / 8; ++t) {
+          const uint32_t v8[8] = {qv[2 * t].x,     qv[2 * t].y,     qv[2 * t].z,     qv[2 * t].w,
+                                  qv[2 * t + 1].x, qv[2 * t + 1].y, qv[2 * t + 1].z, qv[2 * t + 1].w};
+          tmem_st8(tl + qcol + t * 8, v8);
+        }
+        tmem_st_wait();
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&q_full[qb]);
+      return fine;
     };
 
     // jobs with no pages at all (empty prompt and suffixes, some row active)
@@ -534,47 +590,17 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     int gi = 0, pc = 0;
     bool ok = true;
     Job cur;
-    if (b < e && active) cur = job_at(p, gpre, b);
-    int64_t x0 = active ? b : e;
-    while (x0 < e) {
+    const int64_t x_end = in_piece ? e : b;
+    if (b < x_end) {
+      cur = job_at(p, gpre, b);
+      if (!write_q(cur, 0)) ok = false;
+    }
+    for (int64_t x0 = b; x0 < x_end;) {
       const int n_in = (int)(min(e, cur.start + cur.n) - x0);
       const int j = cur.g * p.Hkv + cur.h;
-      const int qb = pc & 1;
-      // ---- this warp's share of its rows' queries -> Q buffer in TMEM ----
-      if (pc >= 2 && ok && !wwait(&q_empty[qb], (uint32_t)((pc >> 1) - 1) & 1u, abort_flag)) ok = false;
-      if (ok) {
-        constexpr int kQChunk = 8;    // uint4 loads in flight (32 registers)
-        const int nld = qcols / 4;    // uint4 loads of this warp's share
-        const bool qrow = r < nq;
-        const uint4* src = nullptr;
-        if (qrow) {
-          const int rr = cur.g * p.rpg + r / gq, hq = cur.h * gq + r % gq;
-          src = reinterpret_cast<const uint4*>(p.q + ((int64_t)rr * p.Hq + hq) * D) + pj * nld;
-        }
-        const uint32_t qcol = kQCol + qb * (D / 2) + pj * qcols;
-#pragma unroll 1
-        for (int t0 = 0; t0 < nld; t0 += kQChunk) {
-          uint4 qv[kQChunk];
-#pragma unroll
-          for (int t = 0; t < kQChunk; ++t)
-            qv[t] = (qrow && t0 + t < nld) ? __ldg(src + t0 + t) : make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-          for (int t = 0; t < kQChunk / 2; ++t) {
-            if (t0 + 2 * t < nld) {
-              const uint32_t v8[8] = {qv[2 * t].x,     qv[2 * t].y,     qv[2 * t].z,     qv[2 * t].w,
-                                      qv[2 * t + 1].x, qv[2 * t + 1].y, qv[2 * t + 1].z, qv[2 * t + 1].w};
-              tmem_st8(tl + qcol + (t0 / 2 + t) * 8, v8);
-            }
-          }
-        }
-        tmem_st_wait();
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&q_full[qb]);
-
       float m_used = -INFINITY, l = 0.f;  // m_used is shared by the W warps of a quarter; l is per warp
-      for (int k0 = 0; k0 < n_in; k0 += kGroupPages) {
+      if (!in_group) gi += (n_in + kGroupPages - 1) / kGroupPages;
+      for (int k0 = 0; in_group && k0 < n_in; k0 += kGroupPages) {
         const int ng = min(kGroupPages, n_in - k0);
         const int sb = gi % kSPBufs, gs = gi % ns;
         if (ok && !wwait(&s_full[sb], (uint32_t)(gi / kSPBufs) & 1u, abort_flag)) ok = false;
@@ -669,32 +695,33 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         if (lane == 0) mbar_arrive(&p_full[sb]);
         ++gi;
       }
+      // ---- the next piece's Q goes in first, so that its QKs overlap this epilogue ----
+      Job nxt = cur;
+      const bool more = x0 + n_in < e;
+      if (more) {
+        nxt = next_job(p, gpre, cur);
+        if (!write_q(nxt, pc + 1)) ok = false;
+      }
       // ---- end of the piece: O is final once the last group's PV completes ----
       const int lg = gi - 1;
       if (ok && !wwait(&p_empty[lg % kSPBufs], (uint32_t)(lg / kSPBufs) & 1u, abort_flag)) ok = false;
       tc_fence_after();
-      // the quarter's row sum over its W warps
-      float Lq = l;
-      if (W > 1) {
+      if (in_group) {
         rsum[pj * kRows + tlane] = l;
-        soft_sync();
-        Lq = rsum[tlane];
-        for (int w = 1; w < W; ++w) Lq += rsum[w * kRows + tlane];
+        if (pj == 0) mfin[tlane] = m_used;
       }
-      // the copies' (m, l) -> the piece's max M and sum L; copy c's O is weighted by 2^(m_c - M)
-      float M = m_used, Ls = Lq, wself = 1.f;
-      if (R > 1) {
-        if (pj == 0) mlx[tlane] = make_float2(m_used, Lq);
-        soft_sync();
-        M = -INFINITY;
-        for (int c2 = 0; c2 < R; ++c2) M = fmaxf(M, mlx[(c2 * qpc + rb) * 32 + lane].x);
-        Ls = 0.f;
-        for (int c2 = 0; c2 < R; ++c2) {
-          const float2 ml = mlx[(c2 * qpc + rb) * 32 + lane];
-          if (ml.x != -INFINITY) Ls += exp2f(ml.x - M) * ml.y;
-        }
-        wself = (m_used == -INFINITY) ? 0.f : exp2f(m_used - M);
+      piece_sync();
+      // the copies' running maxima and row sums -> the piece's max M and sum L;
+      // copy c's O is weighted by 2^(m_c - M)
+      float M = -INFINITY, Ls = 0.f;
+      for (int c2 = 0; c2 < R; ++c2) M = fmaxf(M, mfin[(c2 * qpc + rb) * 32 + lane]);
+      for (int c2 = 0; c2 < R; ++c2) {
+        const int ln = (c2 * qpc + rb) * 32 + lane;
+        float Lc = 0.f;
+        for (int w = 0; w < W; ++w) Lc += rsum[w * kRows + ln];
+        if (mfin[ln] != -INFINITY) Ls += exp2f(mfin[ln] - M) * Lc;
       }
+      const float wself = mfin[tlane] == -INFINITY ? 0.f : exp2f(mfin[tlane] - M);
       const int first = cta_of(cur.start, T, Ceff), last = cta_of(cur.start + cur.n - 1, T, Ceff);
       const bool mine_row = r < nq && cp == 0;
       const int rr = r < nq ? cur.g * p.rpg + r / gq : 0, hq = r < nq ? cur.h * gq + r % gq : 0;
@@ -703,13 +730,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
       // after an abort the piece's outputs are not written (the status word says so)
       const bool out_ok = __all_sync(0xffffffffu, ok && !*abort_flag);
-      // O, 16 columns per round; copies >= 1 pass theirs to copy 0 through shared
-      // memory (double-buffered, so one barrier per round)
-      const int my_stage = ((cp - 1) * qpc + rb) * W + pj;  // (for copies >= 1)
-      const int stage_n = (R - 1) * qpc * W;  // staging rows of 32 lanes x 16 floats per buffer
+      // O, 16 columns per round; copies >= 1 pass theirs to copy 0 through shared memory
+      const int my_stage = ((cp - 1) * qpc + rb) * 4 + pj;  // (for copies >= 1)
 #pragma unroll 1
-      for (int cc = 0; cc < ocols; cc += 16) {
-        const int col = pj * ocols + cc;
+      for (int cc = 0; cc < kEpiCols; cc += 16) {
+        const int col = pj * kEpiCols + cc;
         float o[16];
         if (out_ok) {
           uint32_t raw[16];
@@ -719,17 +744,17 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
           for (int t = 0; t < 16; ++t) o[t] = __uint_as_float(raw[t]) * wself;
         }
         if (R > 1) {
-          float4* sb4 = stage + ((cc / 16) & 1) * (stage_n * 4 * 32);
+          if (cc > 0) piece_sync();  // the previous round's staging has been read
           if (cp > 0 && out_ok) {
 #pragma unroll
             for (int t = 0; t < 4; ++t)
-              sb4[(my_stage * 4 + t) * 32 + lane] = make_float4(o[4 * t], o[4 * t + 1], o[4 * t + 2], o[4 * t + 3]);
+              stage[(my_stage * 4 + t) * 32 + lane] = make_float4(o[4 * t], o[4 * t + 1], o[4 * t + 2], o[4 * t + 3]);
           }
-          soft_sync();
+          piece_sync();
           if (cp == 0 && out_ok) {
 #pragma unroll 1
             for (int c2 = 1; c2 < R; ++c2) {
-              const float4* src4 = sb4 + ((((c2 - 1) * qpc + rb) * W + pj) * 4) * 32 + lane;
+              const float4* src4 = stage + ((((c2 - 1) * qpc + rb) * 4 + pj) * 4) * 32 + lane;
 #pragma unroll
               for (int t = 0; t < 4; ++t) {
                 const float4 v = src4[t * 32];
@@ -765,10 +790,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       } else if (out_ok && pj == 0 && mine_row) {
         p.slot_ml[s_idx * nq + r] = make_float2(M, Ls);  // the merge kernel finishes the job
       }
-      soft_sync();  // the exchange buffers are reused at the next piece
+      piece_sync();  // the exchange buffers are reused at the next piece
       ++pc;
       x0 += n_in;
-      if (x0 < e) cur = next_job(p, gpre, cur);
+      cur = nxt;
     }
   }
   tc_fence_before();
@@ -780,9 +805,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       const int issued = s_issued;
       for (int g = max(0, issued - ns); g < issued; ++g) mbar_wait(&full_bar[g % ns], (g / ns) & 1);
     }
-    if (warp == kMmaWarp && lane == 0) {
-      umma_commit(&mma_done);  // arrives once every MMA this thread issued has completed
-      mbar_wait(&mma_done, 0);
+    if ((warp == kMmaWarp || warp == kPvWarp) && lane == 0) {
+      uint64_t* md = &mma_done[warp - kMmaWarp];
+      umma_commit(md);  // arrives once every MMA this thread issued has completed
+      mbar_wait(md, 0);
     }
     __syncthreads();
   }

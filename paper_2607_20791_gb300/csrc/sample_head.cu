@@ -1,15 +1,21 @@
 // Sample head: the greedy step G_M and the truncated high-temperature sampler
 // S_{T,theta} of Alg. 1, with min-p truncation and a Philox4x32-10 inverse-CDF
-// draw, reading every logit from HBM exactly once.
+// draw.
 //
-// One thread-block cluster of kClusterCtas CTAs handles one row.  Each CTA
-// copies its contiguous slice of the row into shared memory with bulk copies
-// (split into pieces so reduction starts while later pieces are in flight),
-// reduces (max, lowest-index argmax) over its slice, and the CTAs exchange their
-// results through distributed shared memory.  Sample rows then form the min-p
-// cutoff from the row maximum, sum the kept weights of their slice from shared
-// memory (no second HBM read), exchange the slice sums, and the one CTA whose
-// cumulative range contains u * Z scans its slice for the drawn token.
+// One thread-block cluster of kClusterCtas CTAs handles one row; the row is cut
+// into equal contiguous ranges, one per warp of the cluster, and a warp reads
+// its range as stripes of 32 coalesced 16-byte loads (kBatch stripes in flight
+// per lane).  Pass 1 finds the row's max and lowest-index argmax (warp shuffles,
+// shared memory, then distributed shared memory across the cluster).  Probe
+// rows stop there.  Sample rows form the min-p cutoff from the max and, in
+// pass 2, re-read their range (the row was read a moment ago and kept in L2) to
+// sum the kept weights of every stripe (a lane's few elements in index order,
+// then a butterfly across the lanes), keeping the stripe sums in shared memory.
+// The Philox draw gives the target u * Z, and one warp walks the prefix sums in
+// index order -- CTA, warp, stripe -- re-reads that single stripe and finds the
+// lane and the element.  Sums are fp32 with compensation (a few ulp, well inside
+// the 1e-6 of Z within which a draw counts as a boundary case); FP64 is slow on
+// this part, so the only fp64 step is the cutoff's logarithm, once per row.
 #include <cooperative_groups.h>
 
 #include <cmath>
@@ -25,14 +31,14 @@ namespace {
 constexpr int kClusterCtas = 8;
 constexpr int kHeadThreads = 256;
 constexpr int kHeadWarps = kHeadThreads / 32;
-constexpr int kPieces = 4;
-constexpr int kMaxSliceBytes = 200 * 1024;
+constexpr int kBatch = 4;        // 16-byte loads in flight per lane
+constexpr int kMaxStripes = 64;  // stripes per warp whose sums are kept for the draw
 
 struct HeadParams {
   const uint8_t* logits;
   int32_t rows;
   int32_t vocab;
-  int32_t chunk;  // elements per CTA slice (multiple of 16)
+  int32_t spw;  // stripes per warp
   const uint8_t* is_probe;
   const float* temperature;
   const float* min_p;
@@ -45,20 +51,54 @@ struct HeadParams {
   int32_t* dev_status;
 };
 
+// 16 bytes of logits: 4 fp32 or 8 bf16 elements.
 template <typename T>
-struct Elem;
+struct Vec;
 template <>
-struct Elem<float> {
-  static constexpr int kSize = 4;
-  __device__ static float load(const uint8_t* p) { return *reinterpret_cast<const float*>(p); }
-};
-template <>
-struct Elem<__nv_bfloat16> {
-  static constexpr int kSize = 2;
-  __device__ static float load(const uint8_t* p) {
-    return __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(p));
+struct Vec<float> {
+  static constexpr int kN = 4, kSize = 4;
+  static constexpr uint32_t kNegInf = 0xff800000u, kNegInfWord = 0xff800000u;
+  __device__ static float get(const uint4& w, int k) {
+    const uint32_t u = k == 0 ? w.x : k == 1 ? w.y : k == 2 ? w.z : w.w;
+    return __uint_as_float(u);
   }
+  __device__ static uint32_t scalar(const uint8_t* p) { return *reinterpret_cast<const uint32_t*>(p); }
 };
+template <>
+struct Vec<__nv_bfloat16> {
+  static constexpr int kN = 8, kSize = 2;
+  static constexpr uint32_t kNegInf = 0xff80u, kNegInfWord = 0xff80ff80u;
+  __device__ static float get(const uint4& w, int k) {
+    const uint32_t u = (k >> 1) == 0 ? w.x : (k >> 1) == 1 ? w.y : (k >> 1) == 2 ? w.z : w.w;
+    return __uint_as_float((k & 1) ? (u & 0xffff0000u) : (u << 16));
+  }
+  __device__ static uint32_t scalar(const uint8_t* p) { return *reinterpret_cast<const uint16_t*>(p); }
+};
+
+// The kN logits at element i of a row (i a multiple of kN); those at or past
+// `vocab` read as -inf.  kAligned: the row starts 16-byte aligned and holds a
+// whole number of 16-byte vectors.
+template <typename T, bool kAligned>
+__device__ __forceinline__ uint4 load_vec(const uint8_t* row, int64_t i, int32_t vocab, uint64_t policy) {
+  using V = Vec<T>;
+  if (kAligned) {
+    if (i < vocab) return ld_nc_v4_hint(row + i * V::kSize, policy);
+    return make_uint4(V::kNegInfWord, V::kNegInfWord, V::kNegInfWord, V::kNegInfWord);
+  }
+  uint32_t u[4];
+  if (V::kSize == 4) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) u[k] = (i + k < vocab) ? V::scalar(row + (i + k) * 4) : V::kNegInf;
+  } else {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const uint32_t lo = (i + 2 * k < vocab) ? V::scalar(row + (i + 2 * k) * 2) : V::kNegInf;
+      const uint32_t hi = (i + 2 * k + 1 < vocab) ? V::scalar(row + (i + 2 * k + 1) * 2) : V::kNegInf;
+      u[k] = lo | (hi << 16);
+    }
+  }
+  return make_uint4(u[0], u[1], u[2], u[3]);
+}
 
 // Philox4x32-10 (Salmon et al., SC'11): word 0 of the block for (counter, key).
 __device__ __forceinline__ uint32_t philox_word0(uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3,
@@ -86,32 +126,48 @@ __device__ __forceinline__ bool better(float v, int32_t i, float bv, int32_t bi)
 }
 
 struct Shared {
-  uint64_t bar[kPieces];
   float red_v[kHeadWarps];
   int32_t red_i[kHeadWarps];
-  double red_d[kHeadWarps];
+  float red_s[kHeadWarps];
   int32_t red_c[kHeadWarps];
+  float stripe_sum[kHeadWarps][kMaxStripes];
   // published to the cluster
   float cta_max;
   int32_t cta_arg;
-  double cta_sum;
+  float cta_sum;
   int32_t cta_cnt;
   // broadcast within the CTA
   float row_max;
   int32_t row_arg;
-  double target;
-  double cta_base;
-  int32_t claim;
-  int32_t bad;
+  float cut;
 };
 
-template <typename T>
-__global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThreads)
+// Compensated (Kahan) fp32 running sum: the prefix sums of the draw stay within
+// a few ulp of exact without fp64, which is slow on this part.
+struct KSum {
+  float s = 0.f, c = 0.f;
+  __device__ __forceinline__ void add(float x) {
+    const float y = x - c;
+    const float t = s + y;
+    c = (t - s) - y;
+    s = t;
+  }
+  __device__ __forceinline__ float value() const { return s - c; }
+};
+
+// The kept weight of logit l (0 when below the cutoff); the same fp32 steps
+// everywhere, so pass 2 and the draw agree bit for bit.
+__device__ __forceinline__ float kept_weight(float l, float cut, float M, float temp) {
+  return l >= cut ? expf(__fdiv_rn(__fsub_rn(l, M), temp)) : 0.f;
+}
+
+template <typename T, bool kAligned>
+__global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThreads, 5)
     sample_head_kernel(const HeadParams p) {
-  using E = Elem<T>;
-  constexpr int ES = E::kSize;
+  using V = Vec<T>;
+  constexpr int kN = V::kN;
+  constexpr int kStripe = 32 * kN;  // elements per stripe
   __shared__ Shared sh;
-  extern __shared__ __align__(128) uint8_t dyn[];
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = (int)cluster.block_rank();
   const int row = blockIdx.x / kClusterCtas;
@@ -124,87 +180,54 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
     }
     return;
   }
-
-  // ---- slice of the row owned by this CTA ---------------------------------
-  const int32_t e0 = min(p.vocab, rank * p.chunk);
-  const int32_t e1 = min(p.vocab, e0 + p.chunk);
-  const int32_t n = e1 - e0;
-  const uint8_t* gsrc = p.logits + ((int64_t)row * p.vocab + e0) * ES;
-  const uint32_t mis = (uint32_t)(reinterpret_cast<uintptr_t>(gsrc) & 15u);
-  const int32_t head_el = min(n, (int32_t)(((16u - mis) & 15u) / ES));
-  const uint32_t int_bytes = (uint32_t)((n - head_el) * ES) & ~15u;
-  const int32_t int_el = (int32_t)(int_bytes / ES);
-  // sbuf[k] holds element e0 + k; the bulk-copied interior starts 16-byte aligned
-  uint8_t* sbuf = dyn + ((16u - (uint32_t)(head_el * ES)) & 15u);
-  const uint32_t piece = ((int_bytes + kPieces - 1) / kPieces + 15u) & ~15u;
-
+  const uint8_t* rowp = p.logits + (int64_t)row * p.vocab * V::kSize;
+  const int spw = p.spw;
+  // warp w of CTA r reads stripes [(8r + w) spw, (8r + w + 1) spw) of the row
+  auto elem = [&](int w, int s, int k) {
+    return ((int64_t)(rank * kHeadWarps + w) * spw + s) * kStripe + lane * kN + k;
+  };
+  // the row is read again by pass 2 a few microseconds later: pass 1 asks L2 to
+  // keep it, pass 2 (its last full read) lets it go
+  const uint64_t keep_pol = policy_evict_last(), drop_pol = policy_evict_first();
+  // the draw for this row, computed while the logits stream in
+  float u = 0.f;
   if (tid == 0) {
-    for (int k = 0; k < kPieces; ++k) mbar_init(&sh.bar[k], 1);
-    fence_mbar_init();
-  }
-  __syncthreads();
-  if (tid == 0) {
-    for (int k = 0; k < kPieces; ++k) {
-      const uint32_t b = k * piece;
-      if (b >= int_bytes) break;
-      const uint32_t sz = min(piece, int_bytes - b);
-      mbar_arrive_expect_tx(&sh.bar[k], sz);
-      bulk_load(sbuf + head_el * ES + b, gsrc + head_el * ES + b, sz, &sh.bar[k]);
-    }
+    const uint64_t sd = p.seed[row];
+    const uint32_t x0 = philox_word0((uint32_t)p.step, (uint32_t)(p.step >> 32), 0u, 0u, (uint32_t)sd,
+                                     (uint32_t)(sd >> 32));
+    u = (float)(x0 >> 8) * (1.0f / 16777216.0f);  // exact: 24 bits
   }
 
-  // ---- phase 1: max and lowest-index argmax of the slice ---------------------
+  // ---- pass 1: max and lowest-index argmax ----------------------------------
   float bv = -INFINITY;
   int32_t bi = 0x7fffffff;
-  // ragged edges (fewer than 16 bytes each) with plain loads
-  for (int32_t k = tid; k < n - int_el; k += kHeadThreads) {
-    const int32_t idx = (k < head_el) ? k : (head_el + int_el + (k - head_el));
-    const float v = E::load(gsrc + idx * ES);
-    *reinterpret_cast<T*>(sbuf + idx * ES) = *reinterpret_cast<const T*>(gsrc + idx * ES);
-    if (better(v, e0 + idx, bv, bi)) { bv = v; bi = e0 + idx; }
-  }
-  bool timed_out = false;
-  for (int k = 0; k < kPieces; ++k) {
-    const uint32_t b = k * piece;
-    if (b >= int_bytes) break;
-    const uint32_t sz = min(piece, int_bytes - b);
-    // bounded: a copy that never lands is reported, and the later pieces are
-    // still waited for (again bounded) so no copy is in flight at exit
-    if (!mbar_wait(&sh.bar[k], 0)) {
-      timed_out = true;
-      continue;
-    }
-    if (timed_out) continue;
-    const uint8_t* base = sbuf + head_el * ES + b;
-    const int32_t el_base = head_el + (int32_t)(b / ES);
-    for (uint32_t off = tid * 16u; off < sz; off += kHeadThreads * 16u) {
-      const uint4 w = *reinterpret_cast<const uint4*>(base + off);
-      const int32_t i0 = e0 + el_base + (int32_t)(off / ES);
-      if constexpr (ES == 4) {
-        const float v[4] = {__uint_as_float(w.x), __uint_as_float(w.y), __uint_as_float(w.z),
-                            __uint_as_float(w.w)};
+  for (int s0 = 0; s0 < spw; s0 += kBatch) {
+    uint4 w[kBatch];
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
-          if (better(v[j], i0 + j, bv, bi)) { bv = v[j]; bi = i0 + j; }
-      } else {
-        const uint32_t u[4] = {w.x, w.y, w.z, w.w};
+    for (int b = 0; b < kBatch; ++b)
+      if (s0 + b < spw) w[b] = load_vec<T, kAligned>(rowp, elem(warp, s0 + b, 0), p.vocab, keep_pol);
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const float lo = __uint_as_float(u[j] << 16), hi = __uint_as_float(u[j] & 0xffff0000u);
-          if (better(lo, i0 + 2 * j, bv, bi)) { bv = lo; bi = i0 + 2 * j; }
-          if (better(hi, i0 + 2 * j + 1, bv, bi)) { bv = hi; bi = i0 + 2 * j + 1; }
+    for (int b = 0; b < kBatch; ++b) {
+      if (s0 + b >= spw) break;
+      const int32_t base = (int32_t)elem(warp, s0 + b, 0);
+#pragma unroll
+      for (int k = 0; k < kN; ++k) {
+        const float v = V::get(w[b], k);
+        if (v > bv) {  // indices only grow along a lane: strict > keeps the lowest
+          bv = v;
+          bi = base + k;
         }
       }
     }
   }
-  // the row's outputs are invalid after a timeout; the protocol still runs to
-  // its end so that every CTA of the cluster meets the same cluster barriers
-  if (timed_out && tid == 0 && p.dev_status) atomicOr(p.dev_status, RGD_DEV_WAIT_TIMEOUT);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
     const int32_t oi = __shfl_xor_sync(0xffffffffu, bi, o);
-    if (better(ov, oi, bv, bi)) { bv = ov; bi = oi; }
+    if (better(ov, oi, bv, bi)) {
+      bv = ov;
+      bi = oi;
+    }
   }
   if (lane == 0) {
     sh.red_v[warp] = bv;
@@ -215,26 +238,45 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
     float v = sh.red_v[0];
     int32_t i = sh.red_i[0];
     for (int w = 1; w < kHeadWarps; ++w)
-      if (better(sh.red_v[w], sh.red_i[w], v, i)) { v = sh.red_v[w]; i = sh.red_i[w]; }
+      if (better(sh.red_v[w], sh.red_i[w], v, i)) {
+        v = sh.red_v[w];
+        i = sh.red_i[w];
+      }
     sh.cta_max = v;
     sh.cta_arg = i;
   }
-  cluster.sync();  // #1: slice maxima visible to the cluster
-  if (tid == 0) {
+  cluster.sync();  // #1: range maxima visible to the cluster
+  const float temp = p.temperature[row];
+  const float mp = p.min_p[row];
+  if (warp == 0) {
+    // one lane per CTA of the cluster reads its maximum (the remote loads overlap)
     float v = -INFINITY;
     int32_t i = 0x7fffffff;
-    for (int r = 0; r < kClusterCtas; ++r) {
-      const Shared* o = cluster.map_shared_rank(&sh, r);
-      if (better(o->cta_max, o->cta_arg, v, i)) { v = o->cta_max; i = o->cta_arg; }
+    if (lane < kClusterCtas) {
+      const Shared* o = cluster.map_shared_rank(&sh, lane);
+      v = o->cta_max;
+      i = o->cta_arg;
     }
-    sh.row_max = v;
-    sh.row_arg = i;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, v, o);
+      const int32_t oi = __shfl_xor_sync(0xffffffffu, i, o);
+      if (better(ov, oi, v, i)) {
+        v = ov;
+        i = oi;
+      }
+    }
+    if (lane == 0) {
+      sh.row_max = v;
+      sh.row_arg = i;
+      // the min-p cutoff fl32(M + fl32(T ln p_min)); the logarithm in fp64 by one thread
+      const float theta = (mp > 0.0f) ? (float)((double)temp * log((double)mp)) : -INFINITY;
+      sh.cut = __fadd_rn(v, theta);
+    }
   }
   __syncthreads();
   const float M = sh.row_max;
   const int32_t A = sh.row_arg;
-  const float temp = p.temperature[row];
-  const float mp = p.min_p[row];
   const bool greedy = (p.is_probe && p.is_probe[row]) || temp == 0.0f;
   const bool bad = !(temp >= 0.0f) || !isfinite(temp) || !(mp >= 0.0f && mp <= 1.0f) || !isfinite(M) ||
                    A >= p.vocab;
@@ -253,101 +295,156 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
     return;
   }
 
-  // ---- phase 2: min-p cutoff and kept weights of this CTA's slice -------------
-  const float theta = (mp > 0.0f) ? (float)((double)temp * log((double)mp)) : -INFINITY;
-  const float cut = __fadd_rn(M, theta);
-  const int32_t per = (n + kHeadThreads - 1) / kHeadThreads;
-  const int32_t k0 = min(n, tid * per), k1 = min(n, k0 + per);
-  float s = 0.0f, comp = 0.0f;  // Kahan-compensated sum of this thread's kept weights
+  // ---- pass 2: kept weights; the sum of every stripe and of every warp -------
+  const float cut = sh.cut;
+  uint8_t* mask = p.kept_mask ? p.kept_mask + (int64_t)row * p.vocab : nullptr;
+  KSum wsum;  // identical in every lane
   int32_t cnt = 0;
-  uint8_t* mask = p.kept_mask ? p.kept_mask + (int64_t)row * p.vocab + e0 : nullptr;
-  for (int32_t k = k0; k < k1; ++k) {
-    const float l = E::load(sbuf + k * ES);
-    const bool keep = l >= cut;
-    if (mask) mask[k] = keep ? 1 : 0;
-    if (keep) {
-      const float w = expf(__fdiv_rn(__fsub_rn(l, M), temp));
-      const float y = w - comp;
-      const float t2 = s + y;
-      comp = (t2 - s) - y;
-      s = t2;
-      ++cnt;
+  for (int s0 = 0; s0 < spw; s0 += kBatch) {
+    uint4 w[kBatch];
+#pragma unroll
+    for (int b = 0; b < kBatch; ++b)
+      if (s0 + b < spw) w[b] = load_vec<T, kAligned>(rowp, elem(warp, s0 + b, 0), p.vocab, drop_pol);
+#pragma unroll
+    for (int b = 0; b < kBatch; ++b) {
+      if (s0 + b >= spw) break;
+      const int32_t base = (int32_t)elem(warp, s0 + b, 0);
+      // the lane's kept elements as a bit mask (the padding past the vocabulary reads -inf)
+      uint32_t km = 0;
+#pragma unroll
+      for (int k = 0; k < kN; ++k) km |= (V::get(w[b], k) >= cut && base + k < p.vocab) ? (1u << k) : 0u;
+      cnt += __popc(km);
+      // weights in index order, one kept element per lane at a time: the warp
+      // runs max-over-lanes rounds, not kN, and none where nothing is kept
+      float ls = 0.f;
+      while (km) {
+        const int k = __ffs(km) - 1;
+        km &= km - 1;
+        ls += expf(__fdiv_rn(__fsub_rn(V::get(w[b], k), M), temp));
+      }
+      if (mask) {
+#pragma unroll
+        for (int k = 0; k < kN; ++k)
+          if (base + k < p.vocab) mask[base + k] = V::get(w[b], k) >= cut ? 1 : 0;
+      }
+      float S = ls;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) S += __shfl_xor_sync(0xffffffffu, S, o);
+      if (lane == 0) sh.stripe_sum[warp][s0 + b] = S;
+      wsum.add(S);
     }
   }
-  // exclusive scan of the per-thread sums (double) across the CTA
-  // inclusive warp scan; the exclusive prefix is the previous lane's inclusive
-  // value, so consecutive thread boundaries are monotone and partition exactly
-  double incl = (double)s;
 #pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const double v = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += v;
+  for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+  if (lane == 0) {
+    sh.red_s[warp] = wsum.value();
+    sh.red_c[warp] = cnt;
   }
-  double prev = __shfl_up_sync(0xffffffffu, incl, 1);
-  if (lane == 0) prev = 0.0;
-  int32_t c = cnt;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
-  if (lane == 31) sh.red_d[warp] = incl;
-  if (lane == 0) sh.red_c[warp] = c;
   __syncthreads();
-  double warp_base = 0.0;
-  for (int w = 0; w < warp; ++w) warp_base += sh.red_d[w];
-  const double excl = warp_base + prev;
   if (tid == 0) {
-    double tot = 0.0;
+    KSum t;
     int32_t ct = 0;
     for (int w = 0; w < kHeadWarps; ++w) {
-      tot += sh.red_d[w];
+      t.add(sh.red_s[w]);
       ct += sh.red_c[w];
     }
-    sh.cta_sum = tot;
+    sh.cta_sum = t.value();
     sh.cta_cnt = ct;
   }
-  cluster.sync();  // #2: slice sums visible to the cluster
-  if (tid == 0) {
-    double base = 0.0, mine = 0.0;
-    int32_t count = 0;
-    for (int r = 0; r < kClusterCtas; ++r) {
-      const Shared* o = cluster.map_shared_rank(&sh, r);
-      if (r == rank) mine = base;
-      base += o->cta_sum;
-      count += o->cta_cnt;
-    }
-    const uint64_t sd = p.seed[row];
-    const uint32_t x0 = philox_word0((uint32_t)p.step, (uint32_t)(p.step >> 32), 0u, 0u, (uint32_t)sd,
-                                     (uint32_t)(sd >> 32));
-    const double u = (double)(x0 >> 8) * (1.0 / 16777216.0);
-    const double target = u * base;
-    sh.target = target;
-    sh.cta_base = mine;
-    sh.claim = (mine <= target && target < mine + sh.cta_sum) ? 1 : 0;
-    if (rank == 0 && p.kept_count) p.kept_count[row] = count;
+  cluster.sync();  // #2: range sums visible to the cluster
+
+  // ---- the draw: target u * Z; CTA, warp and stripe by prefix sums in index
+  // order; then the stripe's lanes and the lane's elements --------------------
+  float cs = 0.f;
+  int32_t cc = 0;
+  if (warp == 0 && lane < kClusterCtas) {
+    const Shared* o = cluster.map_shared_rank(&sh, lane);
+    cs = o->cta_sum;
+    cc = o->cta_cnt;
   }
-  __syncthreads();
-  if (sh.claim) {
-    const double target = sh.target;
-    const double lo = sh.cta_base + excl;
-    // the next thread's boundary; the last thread's is the CTA's upper end
-    double hi = __shfl_down_sync(0xffffffffu, lo, 1);
-    if (lane == 31) hi = (warp + 1 < kHeadWarps) ? sh.cta_base + (warp_base + sh.red_d[warp])
-                                                   : sh.cta_base + sh.cta_sum;
-    if (lo <= target && target < hi) {
-      double run = lo;
-      int32_t tok = -1, last = -1;
-      for (int32_t k = k0; k < k1; ++k) {
-        const float l = E::load(sbuf + k * ES);
-        if (l >= cut) {
-          last = k;
-          run += (double)expf(__fdiv_rn(__fsub_rn(l, M), temp));
-          if (run > target) {
-            tok = k;
-            break;
-          }
+  if (warp == 0) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) cc += __shfl_xor_sync(0xffffffffu, cc, o);
+    // every lane forms the same prefix sums over the CTAs in rank order
+    KSum pre;
+    float lo = 0.f, hi = 0.f, mine = 0.f;
+    int last_nz = -1;
+    for (int r = 0; r < kClusterCtas; ++r) {
+      const float v = __shfl_sync(0xffffffffu, cs, r);
+      if (r == rank) {
+        lo = pre.value();
+        mine = v;
+      }
+      pre.add(v);
+      if (r == rank) hi = pre.value();
+      if (v > 0.f) last_nz = r;
+    }
+    const float target = __shfl_sync(0xffffffffu, u, 0) * pre.value();
+    if (lane == 0 && rank == 0 && p.kept_count) p.kept_count[row] = cc;
+    if (mine > 0.f && lo <= target && (target < hi || rank == last_nz)) {
+      // the warp, then the stripe, whose range holds the target (the last nonzero
+      // one if rounding leaves the target past every range)
+      KSum wp;
+      wp.add(lo);
+      int cw = -1;
+      float wbase = 0.f;
+      for (int w = 0; w < kHeadWarps; ++w) {
+        const float v = sh.red_s[w];
+        const float before = wp.value();
+        wp.add(v);
+        if (v > 0.f) {
+          cw = w;
+          wbase = before;
+          if (target < wp.value()) break;
         }
       }
-      if (tok < 0) tok = last;
-      p.token_out[row] = e0 + tok;
+      KSum sp;
+      sp.add(wbase);
+      int cst = -1;
+      float sbase = 0.f;
+      for (int st = 0; st < spw; ++st) {
+        const float v = sh.stripe_sum[cw][st];
+        const float before = sp.value();
+        sp.add(v);
+        if (v > 0.f) {
+          cst = st;
+          sbase = before;
+          if (target < sp.value()) break;
+        }
+      }
+      // (a warp or stripe is always found: a range with a nonzero sum has a
+      // nonzero part; the guard only keeps a broken invariant from reading out of range)
+      if (cw < 0 || cst < 0) cw = cst = 0;
+      // the stripe's lanes: the same weights as pass 2, an inclusive scan in index order
+      const uint4 w = load_vec<T, kAligned>(rowp, elem(cw, cst, 0), p.vocab, drop_pol);
+      float ls = 0.f;
+#pragma unroll
+      for (int k = 0; k < kN; ++k) ls += kept_weight(V::get(w, k), cut, M, temp);
+      float incl = ls;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float v = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += v;
+      }
+      const uint32_t over = __ballot_sync(0xffffffffu, ls > 0.f && sbase + incl > target);
+      const uint32_t kept_lanes = __ballot_sync(0xffffffffu, ls > 0.f);
+      const int L = over ? __ffs(over) - 1 : (kept_lanes ? 31 - __clz(kept_lanes) : 0);
+      int32_t tok = -1;
+      if (lane == L) {
+        float r2 = sbase + (incl - ls);
+        int32_t lk = -1;
+#pragma unroll
+        for (int k = 0; k < kN; ++k) {
+          const float wk = kept_weight(V::get(w, k), cut, M, temp);
+          if (wk > 0.f) {
+            lk = (int32_t)elem(cw, cst, k);
+            r2 += wk;
+            if (r2 > target && tok < 0) tok = lk;
+          }
+        }
+        if (tok < 0) tok = lk;  // rounding put the target past the lane's last kept token
+        p.token_out[row] = tok >= 0 ? tok : A;
+      }
     }
   }
   cluster.sync();  // #3: shared memory stays alive until the cluster is done reading it
@@ -373,23 +470,24 @@ extern "C" int rgd_sample_head(int32_t rows, int32_t vocab, int32_t dtype, const
   RGD_CHECK_ARG(aligned16(logits), "rgd_sample_head: logits must be 16-byte aligned");
   RGD_CHECK_ARG(rows <= 0x7fffffff / kClusterCtas, "rgd_sample_head: too many rows");
   const int es = dtype == RGD_F32 ? 4 : 2;
-  const int32_t chunk = ((vocab + kClusterCtas - 1) / kClusterCtas + 15) & ~15;
-  const int smem = chunk * es + 32;
-  if (chunk * es > kMaxSliceBytes)
-    return set_error(RGD_ERR_UNSUPPORTED, "rgd_sample_head: vocab %d too large (max slice %d bytes)", vocab,
-                     kMaxSliceBytes);
-  HeadParams hp{static_cast<const uint8_t*>(logits), rows, vocab, chunk, is_probe, temperature, min_p, seed,
+  const int per_vec = 16 / es;
+  const int64_t stripe = 32 * per_vec;
+  const int64_t warps = (int64_t)kClusterCtas * kHeadWarps;
+  const int32_t spw = (int32_t)((vocab + stripe * warps - 1) / (stripe * warps));
+  if (spw > kMaxStripes)
+    return set_error(RGD_ERR_UNSUPPORTED, "rgd_sample_head: vocab %d too large (max %lld)", vocab,
+                     (long long)(kMaxStripes * stripe * warps));
+  const bool aligned = ((int64_t)vocab * es) % 16 == 0;
+  HeadParams hp{static_cast<const uint8_t*>(logits), rows, vocab, spw, is_probe, temperature, min_p, seed,
                 step, row_active, token_out, kept_count, kept_mask, dev_status};
   const dim3 grid(rows * kClusterCtas), block(kHeadThreads);
   cudaStream_t st = (cudaStream_t)stream;
   if (dtype == RGD_F32) {
-    static bool done = false;
-    if (int rc = ensure_smem(sample_head_kernel<float>, kMaxSliceBytes + 32, &done)) return rc;
-    sample_head_kernel<float><<<grid, block, smem, st>>>(hp);
+    if (aligned) sample_head_kernel<float, true><<<grid, block, 0, st>>>(hp);
+    else sample_head_kernel<float, false><<<grid, block, 0, st>>>(hp);
   } else {
-    static bool done = false;
-    if (int rc = ensure_smem(sample_head_kernel<__nv_bfloat16>, kMaxSliceBytes + 32, &done)) return rc;
-    sample_head_kernel<__nv_bfloat16><<<grid, block, smem, st>>>(hp);
+    if (aligned) sample_head_kernel<__nv_bfloat16, true><<<grid, block, 0, st>>>(hp);
+    else sample_head_kernel<__nv_bfloat16, false><<<grid, block, 0, st>>>(hp);
   }
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? RGD_OK : cuda_error(e, "sample_head launch");
