@@ -18,6 +18,7 @@ every rank runs its own batch (weak scaling, no collective in the data path).
 from __future__ import annotations
 
 import argparse
+import inspect
 import hashlib
 import json
 import os
@@ -79,7 +80,7 @@ def _kernel_hash():
 def _profiled_traffic():
     """Per-launch DRAM bytes of the attention kernel from the committed ncu summary,
     if it was taken on the current kernel source (else None)."""
-    path = os.path.join(ROOT, "profiles", "attn_split_kernel_llama8b.md")
+    path = os.path.join(ROOT, "profiles", "attn_tc_kernel_llama8b.md")
     try:
         text = open(path).read()
     except OSError:
@@ -270,47 +271,71 @@ def run_ours(args):
         binding.rgd_probe_gate(trie, G, rpg, head.token_out, 1, rpg, case.gate.eos, case.gate.max_len, gstate,
                                gate_active, head.dev_status, stream=stream.cuda_stream)
 
+    # The whole step is one CUDA graph; a timing event recorded inside it (an
+    # "external" event) splits it into attention and sample head + gate.
+    one_graph = "external" in inspect.signature(torch.cuda.Event.__new__).parameters
     with torch.cuda.stream(stream):
         for _ in range(3):  # eager warm-up (also sets kernel attributes before capture)
             attn_call()
             head_gate_call()
         torch.cuda.synchronize()
-        g_attn, g_hg = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g_attn, stream=stream):
-            attn_call()
-        with torch.cuda.graph(g_hg, stream=stream):
-            head_gate_call()
+        if one_graph:
+            ev_mid = torch.cuda.Event(enable_timing=True, external=True)
+            g_step = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g_step, stream=stream):
+                attn_call()
+                ev_mid.record(stream)
+                head_gate_call()
+            graphs = [g_step]
+        else:
+            g_attn, g_hg = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g_attn, stream=stream):
+                attn_call()
+            with torch.cuda.graph(g_hg, stream=stream):
+                head_gate_call()
+            graphs = [g_attn, g_hg]
         torch.cuda.synchronize()
     launches_per_step = 5  # attention, split-job merge, sample head, gate-state reset, gate
 
-    def one_step(ev):
+    def one_step():
+        """Runs one timed step; returns (step, attention, head + gate) in ms."""
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
         flush.fill_(1)
         ev[0].record(stream)
-        g_attn.replay()
-        ev[1].record(stream)
-        g_hg.replay()
-        ev[2].record(stream)
+        if one_graph:
+            g_step.replay()
+            ev[2].record(stream)
+            ev[2].synchronize()  # ev_mid is re-recorded by every replay: read it now
+            mid = ev_mid
+        else:
+            g_attn.replay()
+            ev[1].record(stream)
+            g_hg.replay()
+            ev[2].record(stream)
+            ev[2].synchronize()
+            mid = ev[1]
+        return ev[0].elapsed_time(ev[2]), ev[0].elapsed_time(mid), mid.elapsed_time(ev[2])
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
-            one_step([torch.cuda.Event(enable_timing=True) for _ in range(3)])
+            one_step()
         torch.cuda.synchronize()
 
-    events = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     if world > 1:
         import torch.distributed as dist
         dist.barrier()
     torch.cuda.synchronize()
+    times = []
     with ClockSampler(torch.cuda.current_device()) as clk:
         with torch.cuda.stream(stream):
             for i in range(args.steps):
-                one_step(events[i])
+                times.append(one_step())
         torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
-    step_ms = [ev[0].elapsed_time(ev[2]) for ev in events]
-    attn_ms = [ev[0].elapsed_time(ev[1]) for ev in events]
-    hg_ms = [ev[1].elapsed_time(ev[2]) for ev in events]
+    step_ms = [t[0] for t in times]
+    attn_ms = [t[1] for t in times]
+    hg_ms = [t[2] for t in times]
     mean_step = sum(step_ms) / len(step_ms)
     mean_attn = sum(attn_ms) / len(attn_ms)
     status = int(att.dev_status.item()) | int(head.dev_status.item())
@@ -345,8 +370,8 @@ def run_ours(args):
                 e2e_ev[i - args.warmup][0].record(stream)
             for k, t in pinned.items():
                 dst[k].copy_(t, non_blocking=True)
-            g_attn.replay()
-            g_hg.replay()
+            for g in graphs:
+                g.replay()
             tok_host.copy_(head.token_out, non_blocking=True)
             st_host.copy_(gstate, non_blocking=True)
             if i >= args.warmup:
@@ -375,12 +400,15 @@ def run_ours(args):
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": WORKLOAD, "rows_per_step": rows_per_step, "groups": G,
                        "l2": "flushed between steps (256 MiB write, outside the timed events)",
-                       "timing": "CUDA events per step on the launching stream; step = attention graph + "
-                                 "sample-head/gate graph", "parallelism": f"replicas x{world}"},
+                       "timing": "CUDA events per step on the launching stream around one CUDA graph of the "
+                                 "step (attention, split-job merge, sample head, gate), split by an event "
+                                 "recorded inside it" if one_graph else
+                                 "CUDA events per step around the attention graph and the sample-head/gate graph",
+                       "parallelism": f"replicas x{world}"},
             "step_hbm_gbs": step_gbs, "step_hbm_frac": step_gbs / peak,
             "step_algorithmic_bytes": step_bytes,
             "kernels_ms": {"attention": mean_attn, "sample_head_and_gate": sum(hg_ms) / len(hg_ms)},
-            "roofline": {"bound": "hbm", "kernel": "attn_persistent_kernel<128>", "achieved": attn_gbs,
+            "roofline": {"bound": "hbm", "kernel": "attn_tc_kernel<128> + attn_merge_kernel<128>", "achieved": attn_gbs,
                          "peak": peak, "unit": "GB/s", "frac": attn_gbs / peak, "traffic": traffic,
                          "algorithmic_bytes": attn_bytes, "peak_source": peak_kind},
             "cpu_baseline": cpu,

@@ -60,19 +60,23 @@ namespace {
 constexpr int kPage = 16;
 constexpr int kSoftWarps = 16;                // warps 0-15: softmax / epilogue
 constexpr int kSoftThreads = kSoftWarps * 32;
-constexpr int kProducerWarp = 16;
-constexpr int kMmaWarp = 17;                  // QK issue (and the TMEM allocation)
-constexpr int kPvWarp = 18;                   // PV issue
-constexpr int kAttnThreads = 19 * 32;
+constexpr int kProducerWarp = 16;             // warps 16 and 17: page producers
+constexpr int kProducerWarps = 2;
+constexpr int kMmaWarp = 18;                  // QK issue (and the TMEM allocation)
+constexpr int kPvWarp = 19;                   // PV issue
+constexpr int kAttnThreads = 20 * 32;
 constexpr int kGroupPages = 4;                // pages per S / P buffer (64 tokens)
 constexpr int kMaxSlots = 8;                  // ring slots, one page group each
-constexpr int kSPBufs = 3;                    // S / P buffers in TMEM
+constexpr int kSBufs = 2;                     // S buffers in TMEM (freed once the softmax has read them)
+constexpr int kPBufs = 3;                     // P buffers in TMEM (freed once their PV is done)
 constexpr int kRows = 128;                    // MMA M: query rows per job
 constexpr int kMaxQueries = kRows;            // rows_per_group * Hq / Hkv
 constexpr int kTmemCols = 512;
 constexpr int kOCol = 0;                      // O: columns [0, D)
-constexpr int kSPCol = 128;                   // S / P buffers: 64 columns each
-constexpr int kQCol = kSPCol + kSPBufs * 64;  // Q buffers: D/2 columns each (two bf16 per column)
+constexpr int kSCol = 128;                    // S buffers: 64 fp32 columns each (4 pages x 16 tokens)
+constexpr int kPCol = kSCol + kSBufs * 64;    // P buffers: 32 columns each (4 pages x 16 bf16)
+constexpr int kQCol = kPCol + kPBufs * 32;    // Q buffers: D/2 columns each (two bf16 per column)
+static_assert(kQCol + 2 * 64 <= 512, "TMEM columns");
 // V as the MN-major B operand of PV: the two 64-column halves of a page tile are
 // MN-direction swizzle atoms 2048 B apart, the two 8-token groups K-direction
 // atoms 1024 B apart.
@@ -180,8 +184,8 @@ __device__ __forceinline__ int cta_of(int64_t x, int64_t T, int C) { return (int
 
 // Bounded wait that also gives up as soon as another role has given up.
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag) {
-  if (*abort_flag) return false;
   if (mbar_try_wait(bar, parity)) return true;
+  if (*abort_flag) return false;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
@@ -192,6 +196,24 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
         return false;
       }
     }
+  }
+}
+
+// Bounded wait until *gen >= want (a shared counter another warp raises).
+__device__ __forceinline__ bool wait_slot_gen(int32_t* gen, int32_t want, volatile int32_t* abort_flag) {
+  volatile int32_t* g = gen;
+  if (*g >= want) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 1;; ++i) {
+    if (*g >= want) return true;
+    if ((i & 63u) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        *abort_flag = 1;
+        return false;
+      }
+    }
+    __nanosleep(32);
   }
 }
 
@@ -211,8 +233,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   int32_t* gpre = reinterpret_cast<int32_t*>(smem + L.gpre);
   uint32_t* descs = reinterpret_cast<uint32_t*>(smem + L.desc);
   __shared__ uint64_t full_bar[kMaxSlots], empty_bar[kMaxSlots];
-  __shared__ uint64_t s_full[kSPBufs], p_full[kSPBufs], p_empty[kSPBufs], q_full[2], q_empty[2], o_free, mma_done[2];
+  __shared__ uint64_t s_full[kSBufs], s_empty[kSBufs], p_full[kPBufs], p_empty[kPBufs];
+  __shared__ uint64_t q_full[2], q_empty[2], o_free, mma_done[2];
   __shared__ int32_t s_abort, s_issued, s_wsum[kAttnThreads / 32];
+  __shared__ int32_t s_slot_gen[kMaxSlots];  // the last group that entered each ring slot
   __shared__ uint32_t s_tmem;
   volatile int32_t* abort_flag = &s_abort;
 
@@ -233,8 +257,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       mbar_init(&full_bar[i], kGroupPages);  // one arrival per page position (absent pages of a short group too)
       mbar_init(&empty_bar[i], 1);           // released by an MMA commit once the group's PV is done
     }
-    for (int i = 0; i < kSPBufs; ++i) {
+    for (int i = 0; i < kSBufs; ++i) {
       mbar_init(&s_full[i], 1);
+      mbar_init(&s_empty[i], n_soft);
+    }
+    for (int i = 0; i < kPBufs; ++i) {
       mbar_init(&p_full[i], n_soft);
       mbar_init(&p_empty[i], 1);
     }
@@ -247,6 +274,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     mbar_init(&mma_done[1], 1);
     s_abort = 0;
     s_issued = 0;
+    for (int i = 0; i < kMaxSlots; ++i) s_slot_gen[i] = -1;
     fence_mbar_init();
   }
   if (warp == kMmaWarp) {
@@ -311,6 +339,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   __syncthreads();
   if (c == 0)
     for (int g = tid; g <= p.G; g += kAttnThreads) p.gpre_ws[g] = gpre[g];
+  // the merge kernel may be launched now; it waits for this grid to complete
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int64_t T = (int64_t)p.Hkv * gpre[p.G];
   // pages are divided over Ceff = min(C, T) blocks so that every working block
   // has at least one page (a job's pieces are then exactly the blocks first..last)
@@ -318,95 +348,114 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int64_t b = c < Ceff ? (int64_t)c * T / Ceff : T;
   const int64_t e = c < Ceff ? (int64_t)(c + 1) * T / Ceff : T;
 
-  if (warp == kProducerWarp) {
-    // ============================ producer ============================
-    // The warp resolves 32 consecutive pages at a time, one per lane (job by
-    // binary search in shared memory, then the block-table entry).  Then, group
-    // by group, the lane holding a group's first page waits for its slot (group
-    // g of this block goes to slot g % nslots) and every lane of the group
-    // issues its own page's copies: K as two 2 KiB halves into the group's
-    // half-major K block, V as one box.  Groups go in order, so the slot wait
-    // (for the PV of the group nslots back, issued after the QK of the group
-    // after it) never depends on a page not yet issued.
+  if (warp >= kProducerWarp && warp < kProducerWarp + kProducerWarps) {
+    // ============================ producers ===========================
+    // The block's pages are taken 32 at a time, one per lane; the two producer
+    // warps take alternate rounds, so that one warp's block-table loads overlap
+    // the other's copies, and each issues half the copies.  Both walk every
+    // round to number the groups (group g of this block goes to slot
+    // g % nslots; groups restart at each job piece), which needs only shared
+    // memory.  In its own rounds a warp resolves each page (job by binary
+    // search, then the block-table entry) and then, group by group, the first
+    // lane of the group in the round waits for the slot and every lane of the
+    // group issues its page's copies: K as two 2 KiB halves into the group's
+    // half-major K block, V as one box.  A slot wait (for the PV of the group
+    // nslots back, issued after the QK of the group after it) depends only on
+    // pages of earlier groups, and a warp's waits in a round depend only on
+    // pages of earlier rounds, so neither warp can hold up the other.
+    const int pw = warp - kProducerWarp;
     if (b < e) {
-      if (lane == 0) {
+      if (lane == 0 && pw == 0) {
         prefetch_tensormap(&tmK);
         prefetch_tensormap(&tmV);
       }
       const uint64_t pol = policy_evict_first();
       int gbase = 0;  // groups started before xb
-      int64_t xb = b;
-      while (xb < e) {
+      int rnd = 0;
+      for (int64_t xb = b; xb < e; xb += 32, ++rnd) {
         const int64_t x = xb + lane;
         const bool valid = x < e;
+        const bool mine = (rnd % kProducerWarps) == pw;
         int32_t page = -1, tok = 0, rowsel = -1, hh = 0, jpos = 0, ng = 0;
         if (valid) {
           const Job jb = job_at(p, gpre, x);
-          const int k = (int)(x - jb.start);
           // this block's piece of the job starts at max(b, job start); groups restart there
           const int64_t pstart = max(b, jb.start);
           const int kin = (int)(x - pstart);
           const int npiece = (int)(min(e, jb.start + jb.n) - pstart);
           jpos = kin % kGroupPages;
           ng = min(kGroupPages, npiece - (kin - jpos));
-          const int plen = clamp_len(p.prompt_len[jb.g], p.max_pp);
-          const int ppg = (plen + kPage - 1) / kPage;
-          hh = jb.h;
-          if (k < ppg) {
-            page = __ldg(p.prompt_bt + (int64_t)jb.g * p.max_pp + k);
-            tok = min(kPage, plen - k * kPage);
-          } else {
-            int ks = k - ppg;
-            for (int rr = 0; rr < p.rpg; ++rr) {  // the active row holding suffix page ks
-              const int r = jb.g * p.rpg + rr;
-              const int slen = row_on(p, r) ? clamp_len(p.suffix_len[r], p.max_sp) : 0;
-              const int np = (slen + kPage - 1) / kPage;
-              if (ks < np) {
-                page = __ldg(p.suffix_bt + (int64_t)r * p.max_sp + ks);
-                tok = min(kPage, slen - ks * kPage);
-                rowsel = rr;
-                break;
+          if (mine) {
+            const int k = (int)(x - jb.start);
+            const int plen = clamp_len(p.prompt_len[jb.g], p.max_pp);
+            const int ppg = (plen + kPage - 1) / kPage;
+            hh = jb.h;
+            if (k < ppg) {
+              page = __ldg(p.prompt_bt + (int64_t)jb.g * p.max_pp + k);
+              tok = min(kPage, plen - k * kPage);
+            } else {
+              int ks = k - ppg;
+              for (int rr = 0; rr < p.rpg; ++rr) {  // the active row holding suffix page ks
+                const int r = jb.g * p.rpg + rr;
+                const int slen = row_on(p, r) ? clamp_len(p.suffix_len[r], p.max_sp) : 0;
+                const int np = (slen + kPage - 1) / kPage;
+                if (ks < np) {
+                  page = __ldg(p.suffix_bt + (int64_t)r * p.max_sp + ks);
+                  tok = min(kPage, slen - ks * kPage);
+                  rowsel = rr;
+                  break;
+                }
+                ks -= np;
               }
-              ks -= np;
             }
           }
         }
         const bool start = valid && jpos == 0;
         const uint32_t starts = __ballot_sync(0xffffffffu, start);
-        const uint32_t le = 0xffffffffu >> (31 - lane);
-        const int gidx = gbase + __popc(starts & le) - 1;  // lane 0 may continue the last round's group
-        const int g0 = __shfl_sync(0xffffffffu, gidx, 0);
-        const int g1 = __shfl_sync(0xffffffffu, gidx, 31 - __clz(__ballot_sync(0xffffffffu, valid)));
-        const int gs = gidx % ns;
-        bool aborted = false;
-        for (int gq = g0; gq <= g1; ++gq) {
-          const bool in = valid && gidx == gq;
-          int stop = 0;
-          if (in && start && gq >= ns &&
-              !wait_or_abort(&empty_bar[gs], (uint32_t)((gq / ns) - 1) & 1u, abort_flag))
-            stop = 1;
-          if (__any_sync(0xffffffffu, stop != 0)) {
-            aborted = true;
-            break;
-          }
-          if (in) {
-            int32_t y = -2 * kPage;  // fully out of bounds: the TMA fills zeros
-            if (page >= 0 && page < p.num_pages) y = (page * p.Hkv + hh) * kPage;
-            else flag(p.dev_status, RGD_DEV_BAD_PAGE);
-            descs[gs * kGroupPages + jpos] = (uint32_t)tok | ((uint32_t)(rowsel & 0xffff) << 16);
-            uint8_t* sl = smem + gs * kSlot;
-            mbar_arrive_expect_tx(&full_bar[gs], kStage);
-            if (jpos == ng - 1 && ng < kGroupPages) mbar_arrive_cnt(&full_bar[gs], kGroupPages - ng);
+        if (mine) {
+          const uint32_t le = 0xffffffffu >> (31 - lane);
+          const int gidx = gbase + __popc(starts & le) - 1;  // lane 0 may continue the last round's group
+          const int g0 = __shfl_sync(0xffffffffu, gidx, 0);
+          const int g1 = __shfl_sync(0xffffffffu, gidx, 31 - __clz(__ballot_sync(0xffffffffu, valid)));
+          const int gs = gidx % ns;
+          bool aborted = false;
+          for (int gq = g0; gq <= g1; ++gq) {
+            const bool in = valid && gidx == gq;
+            // the group's first lane in this round waits for the slot: first until
+            // the slot's previous group has entered it (the other warp may still be
+            // behind), so that the parity wait on its release is never two phases
+            // ahead, then for that release
+            const bool lead = in && (start || lane == 0);
+            int stop = 0;
+            if (lead && gq >= ns &&
+                (!wait_slot_gen(&s_slot_gen[gs], gq - ns, abort_flag) ||
+                 !wait_or_abort(&empty_bar[gs], (uint32_t)((gq / ns) - 1) & 1u, abort_flag)))
+              stop = 1;
+            if (__any_sync(0xffffffffu, stop != 0)) {
+              aborted = true;
+              break;
+            }
+            if (in) {
+              int32_t y = -2 * kPage;  // fully out of bounds: the TMA fills zeros
+              if (page >= 0 && page < p.num_pages) y = (page * p.Hkv + hh) * kPage;
+              else flag(p.dev_status, RGD_DEV_BAD_PAGE);
+              descs[gs * kGroupPages + jpos] = (uint32_t)tok | ((uint32_t)(rowsel & 0xffff) << 16);
+              uint8_t* sl = smem + gs * kSlot;
+              mbar_arrive_expect_tx(&full_bar[gs], kStage);
+              if (jpos == ng - 1 && ng < kGroupPages) mbar_arrive_cnt(&full_bar[gs], kGroupPages - ng);
 #pragma unroll
-            for (int hf = 0; hf < kHalves; ++hf)
-              tma_load_3d_hint(sl + hf * (kGroupPages * 2048) + jpos * 2048, &tmK, &full_bar[gs], 0, y, hf, pol);
-            tma_load_3d_hint(sl + kVOff + jpos * kTile, &tmV, &full_bar[gs], 0, y, 0, pol);
-            if (start) s_issued = gq + 1;
+              for (int hf = 0; hf < kHalves; ++hf)
+                tma_load_3d_hint(sl + hf * (kGroupPages * 2048) + jpos * 2048, &tmK, &full_bar[gs], 0, y, hf, pol);
+              tma_load_3d_hint(sl + kVOff + jpos * kTile, &tmV, &full_bar[gs], 0, y, 0, pol);
+              if (start) {
+                atomicMax(&s_issued, gq + 1);
+                atomicMax(&s_slot_gen[gs], gq);
+              }
+            }
           }
+          if (aborted) break;
         }
-        if (aborted) break;
         gbase += __popc(starts);
-        xb += 32;
       }
     }
   } else if (warp == kMmaWarp) {
@@ -431,21 +480,21 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         const uint32_t qa = tmem + kQCol + qb * (D / 2);
         for (int k0 = 0; k0 < n_in; k0 += kGroupPages) {
           const int ng = min(kGroupPages, n_in - k0);
-          const int sb = gi % kSPBufs;
+          const int sb = gi % kSBufs;
           const int gs = gi % ns;
           if (!wait_or_abort(&full_bar[gs], (uint32_t)(gi / ns) & 1u, abort_flag)) {
             ok = false;
             break;
           }
-          // the S / P buffer is free once the PV of the group that used it last is done
-          if (gi >= kSPBufs && !wait_or_abort(&p_empty[sb], (uint32_t)((gi / kSPBufs) - 1) & 1u, abort_flag)) {
+          // the S buffer is free once the softmax has read the group that used it last
+          if (gi >= kSBufs && !wait_or_abort(&s_empty[sb], (uint32_t)((gi / kSBufs) - 1) & 1u, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after();
           const uint32_t idesc_qk = idesc_bf16_f32(kRows, kPage * ng, 0, 0);
           const uint64_t kg = k_d + (uint64_t)((gs * kSlot) >> 4);
-          const uint32_t dcol = tmem + kSPCol + sb * 64;
+          const uint32_t dcol = tmem + kSCol + sb * 64;
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk)
             umma_bf16_tmem_a(dcol, qa + kk * 8,
@@ -475,9 +524,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         const int n_in = (int)(min(e, cur.start + cur.n) - x0);
         for (int k0 = 0; k0 < n_in; k0 += kGroupPages) {
           const int ng = min(kGroupPages, n_in - k0);
-          const int pb = gi % kSPBufs;
+          const int pb = gi % kPBufs;
           const int gs = gi % ns;
-          if (!wait_or_abort(&p_full[pb], (uint32_t)(gi / kSPBufs) & 1u, abort_flag)) {
+          if (!wait_or_abort(&p_full[pb], (uint32_t)(gi / kPBufs) & 1u, abort_flag)) {
             ok = false;
             break;
           }
@@ -489,7 +538,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 #pragma unroll
           for (int j = 0; j < kGroupPages; ++j) {
             if (j < ng)
-              umma_bf16_tmem_a(tmem + kOCol, tmem + kSPCol + pb * 64 + j * 8,
+              umma_bf16_tmem_a(tmem + kOCol, tmem + kPCol + pb * 32 + j * 8,
                                v_d + (uint64_t)((gs * kSlot + kVOff + j * kTile) >> 4), kIdescPV,
                                (k0 == 0 && j == 0) ? 0u : 1u);
           }
@@ -584,6 +633,15 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       }
     }
 
+    // P columns of pages this warp's copy does not handle must read 0 in its
+    // lanes: they are never written after this
+    if (in_group) {
+      const uint32_t zero[16] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+#pragma unroll
+      for (int c0 = 0; c0 < kPBufs * 32; c0 += 16) tmem_st16(tl + kPCol + c0, zero);
+      tmem_st_wait();
+    }
+
     // These warps never leave their loops early: the loop structure is the same
     // for all of them, so every named barrier is reached even after an abort
     // (waits then return at once and the work is skipped).
@@ -602,12 +660,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       if (!in_group) gi += (n_in + kGroupPages - 1) / kGroupPages;
       for (int k0 = 0; in_group && k0 < n_in; k0 += kGroupPages) {
         const int ng = min(kGroupPages, n_in - k0);
-        const int sb = gi % kSPBufs, gs = gi % ns;
-        if (ok && !wwait(&s_full[sb], (uint32_t)(gi / kSPBufs) & 1u, abort_flag)) ok = false;
-        const bool has = ok && jp < ng;
-        tc_fence_after();
+        const int sb = gi % kSBufs, pb = gi % kPBufs, gs = gi % ns;
+        const bool has = jp < ng;
         int tok = 0, sel = -1;
-        if (has) {
+        if (has && ok) {
           // this page's descriptor; the producer's write is ordered by the full barrier
           if (wwait(&full_bar[gs], (uint32_t)(gi / ns) & 1u, abort_flag)) {
             const uint32_t dsc = descs[gs * kGroupPages + jp];
@@ -617,34 +673,33 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             ok = false;
           }
         }
+        if (ok && !wwait(&s_full[sb], (uint32_t)(gi / kSBufs) & 1u, abort_flag)) ok = false;
+        tc_fence_after();
         float sc[kPage];
 #pragma unroll
         for (int t = 0; t < kPage; ++t) sc[t] = -INFINITY;
-        const uint32_t scol = kSPCol + sb * 64;
         if (has && ok) {
           uint32_t raw[16];
-          tmem_ld16(tl + scol + jp * kPage, raw);
+          tmem_ld16(tl + kSCol + sb * 64 + jp * kPage, raw);
           tmem_ld_wait();
 #pragma unroll
           for (int t = 0; t < kPage; ++t) sc[t] = __uint_as_float(raw[t]);
         }
+        // S is in registers: its buffer can take the group after next
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&s_empty[sb]);
         // masks: token count of the page, and a suffix page is visible to one row only
         const bool rowok = has && ok && rloc >= 0 && (sel < 0 || sel == rloc);
-        float mx = -INFINITY;
 #pragma unroll
-        for (int t = 0; t < kPage; ++t) {
-          const float v = (rowok && t < tok) ? sc[t] * p.scale_log2 : -INFINITY;
-          sc[t] = v;
-          mx = fmaxf(mx, v);
-        }
+        for (int t = 0; t < kPage; ++t) sc[t] = (rowok && t < tok) ? sc[t] * p.scale_log2 : -INFINITY;
+        float mx = fmaxf(fmaxf(fmaxf(fmaxf(sc[0], sc[1]), fmaxf(sc[2], sc[3])), fmaxf(fmaxf(sc[4], sc[5]), fmaxf(sc[6], sc[7]))),
+                         fmaxf(fmaxf(fmaxf(sc[8], sc[9]), fmaxf(sc[10], sc[11])), fmaxf(fmaxf(sc[12], sc[13]), fmaxf(sc[14], sc[15]))));
         if (W > 1) {
-          // the group's row max over the quarter's page slots; the barrier also
-          // orders every warp's S reads before the P writes that overwrite them
+          // the group's row max over the quarter's page slots
           float* rm = rmax + (gi & 1) * 4 * kRows;
           rm[pj * kRows + tlane] = mx;
-          tc_fence_before();
           soft_sync();
-          tc_fence_after();
           mx = rm[tlane];
           for (int w = 1; w < W; ++w) mx = fmaxf(mx, rm[w * kRows + tlane]);
         }
@@ -653,7 +708,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
           const float nm = need ? mx : m_used;
           const float f = (m_used == -INFINITY) ? 0.f : exp2f(m_used - nm);
           const int pg = gi - 1;
-          if (k0 > 0 && ok && !wwait(&p_empty[pg % kSPBufs], (uint32_t)(pg / kSPBufs) & 1u, abort_flag)) ok = false;
+          if (k0 > 0 && ok && !wwait(&p_empty[pg % kPBufs], (uint32_t)(pg / kPBufs) & 1u, abort_flag)) ok = false;
           if (k0 > 0 && ok) {
             // O holds this piece's earlier groups: the last PV is done; rescale this warp's columns
             tc_fence_after();
@@ -672,27 +727,27 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
           l *= f;
           m_used = nm;
         }
+        // P = 2^(s - m) (ex2 of -inf is +0: masked tokens give 0)
         const float ref = (m_used == -INFINITY) ? 0.f : m_used;
+        float pv[kPage];
+#pragma unroll
+        for (int t = 0; t < kPage; ++t) pv[t] = ex2_approx(sc[t] - ref);
         uint32_t pk[kPage / 2];
 #pragma unroll
-        for (int t = 0; t < kPage; t += 2) {
-          const float p0 = sc[t] == -INFINITY ? 0.f : exp2f(sc[t] - ref);
-          const float p1 = sc[t + 1] == -INFINITY ? 0.f : exp2f(sc[t + 1] - ref);
-          l += p0 + p1;
-          pk[t / 2] = pack_bf16x2(p0, p1);
+        for (int t = 0; t < kPage; t += 2) pk[t / 2] = pack_bf16x2(pv[t], pv[t + 1]);
+        l += ((((pv[0] + pv[1]) + (pv[2] + pv[3])) + ((pv[4] + pv[5]) + (pv[6] + pv[7]))) +
+              (((pv[8] + pv[9]) + (pv[10] + pv[11])) + ((pv[12] + pv[13]) + (pv[14] + pv[15]))));
+        // the P buffer is free once the PV of the group that used it last is done
+        const int pq = gi - kPBufs;
+        if (pq >= 0 && ok && !wwait(&p_empty[pb], (uint32_t)(pq / kPBufs) & 1u, abort_flag)) ok = false;
+        if (has && ok) {
+          tc_fence_after();
+          tmem_st8(tl + kPCol + pb * 32 + jp * 8, pk);  // P of this page (the other copies' pages stay 0)
+          tmem_st_wait();
         }
-        if (has && ok) tmem_st8(tl + scol + jp * 8, pk);  // P of this page, over its S columns
-        if (R > 1 && pj == 0 && ok) {
-          // the other copies' pages contribute nothing to this copy's O
-          const uint32_t zero[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
-#pragma unroll
-          for (int jj = 0; jj < kGroupPages; ++jj)
-            if (jj < ng && jj % R != cp) tmem_st8(tl + scol + jj * 8, zero);
-        }
-        tmem_st_wait();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&p_full[sb]);
+        if (lane == 0) mbar_arrive(&p_full[pb]);
         ++gi;
       }
       // ---- the next piece's Q goes in first, so that its QKs overlap this epilogue ----
@@ -704,7 +759,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       }
       // ---- end of the piece: O is final once the last group's PV completes ----
       const int lg = gi - 1;
-      if (ok && !wwait(&p_empty[lg % kSPBufs], (uint32_t)(lg / kSPBufs) & 1u, abort_flag)) ok = false;
+      if (ok && !wwait(&p_empty[lg % kPBufs], (uint32_t)(lg / kPBufs) & 1u, abort_flag)) ok = false;
       tc_fence_after();
       if (in_group) {
         rsum[pj * kRows + tlane] = l;
@@ -825,6 +880,10 @@ constexpr int kMergeThreads = 256;
 
 template <int D>
 __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnParams p) {
+  // launched as a programmatic dependent of the attention kernel: its launch
+  // overlaps that kernel's tail, and this wait returns once it has completed
+  // and its writes are visible
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int j = blockIdx.x;
   const int g = j / p.Hkv, h = j % p.Hkv;
   const int32_t* gp = p.gpre_ws;
@@ -837,27 +896,49 @@ __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnPar
   if (first == last) return;
   const int nq = p.nq, gq = p.gq;
   constexpr int kChunks = D / 4;
+  constexpr int kP = 4;  // pieces whose loads are issued together
   for (int item = threadIdx.x; item < nq * kChunks; item += kMergeThreads) {
     const int i = item / kChunks, c4 = item % kChunks;
     const int r = g * p.rpg + i / gq, hq = h * gq + i % gq;
     if (!row_on(p, r)) continue;
-    float M = -INFINITY;
-    for (int cc = first; cc <= last; ++cc) M = fmaxf(M, p.slot_ml[((int64_t)cc + j) * nq + i].x);
+    float M = -INFINITY, Ls = 0.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    float Ls = 0.f;
-    if (M != -INFINITY) {
-      for (int cc = first; cc <= last; ++cc) {
-        const int64_t si = ((int64_t)cc + j) * nq + i;
-        const float2 ml = p.slot_ml[si];
-        if (ml.y == 0.f) continue;
-        const float w = exp2f(ml.x - M);
-        Ls += w * ml.y;
-        const float4 v = reinterpret_cast<const float4*>(p.slot_o + si * D)[c4];
-        acc.x += w * v.x;
-        acc.y += w * v.y;
-        acc.z += w * v.z;
-        acc.w += w * v.w;
+    for (int c0 = first; c0 <= last; c0 += kP) {
+      float2 ml[kP];
+      float4 v[kP];
+#pragma unroll
+      for (int t = 0; t < kP; ++t) {
+        if (c0 + t <= last) {
+          const int64_t si = ((int64_t)(c0 + t) + j) * nq + i;
+          ml[t] = p.slot_ml[si];
+          v[t] = reinterpret_cast<const float4*>(p.slot_o + si * D)[c4];
+        } else {
+          ml[t] = make_float2(-INFINITY, 0.f);
+        }
       }
+      // online merge: the running (M, L, acc) absorbs up to kP pieces at once
+      float Mn = M;
+#pragma unroll
+      for (int t = 0; t < kP; ++t)
+        if (ml[t].y != 0.f) Mn = fmaxf(Mn, ml[t].x);
+      if (Mn == -INFINITY) continue;
+      const float f = (M == -INFINITY) ? 0.f : exp2f(M - Mn);
+      Ls *= f;
+      acc.x *= f;
+      acc.y *= f;
+      acc.z *= f;
+      acc.w *= f;
+#pragma unroll
+      for (int t = 0; t < kP; ++t) {
+        if (ml[t].y == 0.f) continue;
+        const float w = exp2f(ml[t].x - Mn);
+        Ls += w * ml[t].y;
+        acc.x += w * v[t].x;
+        acc.y += w * v[t].y;
+        acc.z += w * v[t].z;
+        acc.w += w * v[t].w;
+      }
+      M = Mn;
     }
     const float iv = Ls > 0.f ? 1.f / Ls : 0.f;
     uint2 pk;
@@ -866,6 +947,22 @@ __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnPar
     reinterpret_cast<uint2*>(p.out + ((int64_t)r * p.Hq + hq) * D)[c4] = pk;
     if (p.lse && c4 == 0) p.lse[(int64_t)r * p.Hq + hq] = Ls > 0.f ? (M + log2f(Ls)) * kLn2 : -INFINITY;
   }
+}
+
+// The merge kernel follows the attention kernel as a programmatic dependent.
+template <int D>
+cudaError_t launch_merge(const AttnParams& p, int J, cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(J);
+  cfg.blockDim = dim3(kMergeThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, attn_merge_kernel<D>, p);
 }
 
 // ---------------------------------------------------------------------------
@@ -1038,12 +1135,14 @@ extern "C" int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf1
     static bool done = false;
     if (int rc = ensure_smem(attn_tc_kernel<128>, kSmemLimit, &done)) return rc;
     attn_tc_kernel<128><<<pl.C, kAttnThreads, pl.smem.total, st>>>(tmK, tmV, p);
-    attn_merge_kernel<128><<<pl.J, kMergeThreads, 0, st>>>(p);
+    if (cudaError_t e = cudaGetLastError(); e != cudaSuccess) return cuda_error(e, "attention launch");
+    if (cudaError_t e = launch_merge<128>(p, pl.J, st); e != cudaSuccess) return cuda_error(e, "merge launch");
   } else {
     static bool done = false;
     if (int rc = ensure_smem(attn_tc_kernel<64>, kSmemLimit, &done)) return rc;
     attn_tc_kernel<64><<<pl.C, kAttnThreads, pl.smem.total, st>>>(tmK, tmV, p);
-    attn_merge_kernel<64><<<pl.J, kMergeThreads, 0, st>>>(p);
+    if (cudaError_t e = cudaGetLastError(); e != cudaSuccess) return cuda_error(e, "attention launch");
+    if (cudaError_t e = launch_merge<64>(p, pl.J, st); e != cudaSuccess) return cuda_error(e, "merge launch");
   }
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? RGD_OK : cuda_error(e, "attention launch");
