@@ -58,25 +58,37 @@ namespace rgd {
 namespace {
 
 constexpr int kPage = 16;
-constexpr int kSoftWarps = 16;                // warps 0-15: softmax / epilogue
-constexpr int kSoftThreads = kSoftWarps * 32;
-constexpr int kProducerWarp = 16;             // warps 16 and 17: page producers
 constexpr int kProducerWarps = 2;
-constexpr int kMmaWarp = 18;                  // QK issue (and the TMEM allocation)
-constexpr int kPvWarp = 19;                   // PV issue
-constexpr int kAttnThreads = 20 * 32;
+
+// Warp roles of the attention kernel for R copies of the job's queries in the
+// 128 TMEM lanes (R = 4 / the lane quarters one copy spans).  Each used lane
+// quarter gets W = 4 / R softmax warps (one page of a group each) and, when
+// R > 1, one epilogue warp; then come two producers, the QK issuer and the PV
+// issuer.  Fewer warps leave each more registers (384 threads at R = 4).
+template <int R>
+struct Roles {
+  static constexpr int kW = 4 / R;                   // softmax warps per quarter
+  static constexpr int kNE = R > 1 ? 1 : 0;          // spare epilogue warps per quarter
+  static constexpr int kSoft = 4 * (kW + kNE);       // softmax and epilogue warps
+  static constexpr int kProducer = kSoft;            // kProducerWarps page producers
+  static constexpr int kMma = kSoft + kProducerWarps;  // QK issue (and the TMEM allocation)
+  static constexpr int kPv = kMma + 1;               // PV issue
+  static constexpr int kThreads = (kPv + 1) * 32;
+};
+constexpr int kMaxAttnWarps = Roles<1>::kThreads / 32;
 constexpr int kGroupPages = 4;                // pages per S / P buffer (64 tokens)
 constexpr int kMaxSlots = 8;                  // ring slots, one page group each
 constexpr int kSBufs = 2;                     // S buffers in TMEM (freed once the softmax has read them)
-constexpr int kPBufs = 3;                     // P buffers in TMEM (freed once their PV is done)
+constexpr int kPBufs = 2;                     // P buffers in TMEM (freed once their PV is done)
 constexpr int kRows = 128;                    // MMA M: query rows per job
 constexpr int kMaxQueries = kRows;            // rows_per_group * Hq / Hkv
 constexpr int kTmemCols = 512;
-constexpr int kOCol = 0;                      // O: columns [0, D)
-constexpr int kSCol = 128;                    // S buffers: 64 fp32 columns each (4 pages x 16 tokens)
+constexpr int kOCol = 0;                      // O: two buffers (alternate job pieces) of D columns
+constexpr int kOStride = 128;
+constexpr int kSCol = 2 * kOStride;           // S buffers: 64 fp32 columns each (4 pages x 16 tokens)
 constexpr int kPCol = kSCol + kSBufs * 64;    // P buffers: 32 columns each (4 pages x 16 bf16)
-constexpr int kQCol = kPCol + kPBufs * 32;    // Q buffers: D/2 columns each (two bf16 per column)
-static_assert(kQCol + 2 * 64 <= 512, "TMEM columns");
+constexpr int kQCol = kPCol + kPBufs * 32;    // Q: D/2 columns (two bf16 per column)
+static_assert(kQCol + 64 <= 512, "TMEM columns");
 // V as the MN-major B operand of PV: the two 64-column halves of a page tile are
 // MN-direction swizzle atoms 2048 B apart, the two 8-token groups K-direction
 // atoms 1024 B apart.
@@ -107,7 +119,7 @@ struct AttnParams {
 // Shared-memory carve-up (identical on host and device).  The ring is 1024-byte
 // aligned: the 128-byte swizzle repeats every 8 rows of 128 bytes.
 struct SmemLayout {
-  int ring, red, gpre, gact, desc, total;
+  int ring, red, gpre, gact, desc, rowbits, total;
 };
 
 __host__ __device__ inline int align_up(int x, int a) { return (x + a - 1) / a * a; }
@@ -122,15 +134,17 @@ __host__ __device__ constexpr int slot_bytes() {
 }
 
 template <int D>
-__host__ __device__ inline SmemLayout smem_layout(int nslots, int G) {
+__host__ __device__ inline SmemLayout smem_layout(int nslots, int G, int R) {
   SmemLayout L;
   L.ring = 0;
   L.red = nslots * slot_bytes<D>();
-  // row-max exchange (2 buffers), row-sum exchange, per-lane running max, O staging
-  L.gpre = L.red + (3 * 4 * kRows + kRows + 12 * 4 * 32 * 4) * 4;
+  // row-max exchange (2 buffers), row sums and running maxima of 2 pieces, O
+  // staging for the copies >= 1 (at most 3 warps x 16 columns x 32 lanes)
+  L.gpre = L.red + (2 * 4 * kRows + 2 * 4 * kRows + 2 * kRows + 3 * 4 * 32 * 4) * 4;
   L.gact = align_up(L.gpre + (G + 1) * 4, 16);
   L.desc = align_up(L.gact + G * 4, 16);
-  L.total = align_up(L.desc + nslots * kGroupPages * 4, 16) + 1024;  // + slack for the 1024-byte aligned base
+  L.rowbits = align_up(L.desc + nslots * kGroupPages * 4, 16);  // one bit per row: active
+  L.total = align_up(L.rowbits + (R + 31) / 32 * 4, 16) + 1024;  // + slack for the 1024-byte aligned base
   return L;
 }
 
@@ -183,12 +197,14 @@ __device__ Job next_job(const AttnParams& p, const int32_t* gpre, Job j) {
 __device__ __forceinline__ int cta_of(int64_t x, int64_t T, int C) { return (int)(((x + 1) * C - 1) / T); }
 
 // Bounded wait that also gives up as soon as another role has given up.
+// A waiting thread sleeps inside try_wait (woken when the phase completes), so
+// warps parked on a barrier take no issue slots from the working ones.
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag) {
   if (mbar_try_wait(bar, parity)) return true;
   if (*abort_flag) return false;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
+    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
     if ((i & 63u) == 0) {
       if (*abort_flag) return false;
       if (globaltimer_ns() - t0 > kWaitLimitNs) {
@@ -217,8 +233,8 @@ __device__ __forceinline__ bool wait_slot_gen(int32_t* gen, int32_t want, volati
   }
 }
 
-template <int D>
-__global__ void __launch_bounds__(kAttnThreads, 1)
+template <int D, int R>
+__global__ void __launch_bounds__(Roles<R>::kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                    const AttnParams p) {
   constexpr int kTile = kPage * D * 2;      // one K or V page-head tile
@@ -229,13 +245,18 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   constexpr uint32_t kIdescPV = idesc_bf16_f32(kRows, D, 0, 1);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const SmemLayout L = smem_layout<D>(p.nslots, p.G);
+  const SmemLayout L = smem_layout<D>(p.nslots, p.G, p.G * p.rpg);
+  uint32_t* rowbits = reinterpret_cast<uint32_t*>(smem + L.rowbits);
   int32_t* gpre = reinterpret_cast<int32_t*>(smem + L.gpre);
   uint32_t* descs = reinterpret_cast<uint32_t*>(smem + L.desc);
   __shared__ uint64_t full_bar[kMaxSlots], empty_bar[kMaxSlots];
   __shared__ uint64_t s_full[kSBufs], s_empty[kSBufs], p_full[kPBufs], p_empty[kPBufs];
-  __shared__ uint64_t q_full[2], q_empty[2], o_free, mma_done[2];
-  __shared__ int32_t s_abort, s_issued, s_wsum[kAttnThreads / 32];
+  __shared__ uint64_t q_full, q_empty, o_full[2], o_free[2], ml_full[2], ml_empty[2], mma_done[2];
+  using Rl = Roles<R>;
+  constexpr int kAttnThreads = Rl::kThreads;
+  constexpr int kSoftThreads = Rl::kSoft * 32;
+  constexpr int kProducerWarp = Rl::kProducer, kMmaWarp = Rl::kMma, kPvWarp = Rl::kPv;
+  __shared__ int32_t s_abort, s_issued, s_wsum[kMaxAttnWarps];
   __shared__ int32_t s_slot_gen[kMaxSlots];  // the last group that entered each ring slot
   __shared__ uint32_t s_tmem;
   volatile int32_t* abort_flag = &s_abort;
@@ -246,11 +267,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const uint32_t sbase = smem_u32(smem);
   // The queries fill qpc TMEM lane quarters and are held R times; the softmax
   // warps of unused quarters sit out, and the barriers count the active ones.
-  const int qpc = (p.nq + 31) / 32;         // lane quarters one copy of the queries spans
-  const int R = 4 / qpc;                    // copies of the queries in the 128 lanes
-  const int W = kGroupPages / R;            // softmax warps per quarter (pages per copy and group)
+  const int qpc = (p.nq + 31) / 32;         // lane quarters one copy of the queries spans (4 / R, or 3)
+  constexpr int W = Rl::kW;                 // softmax warps per quarter (pages per copy and group)
+  constexpr bool side = Rl::kNE > 0;        // a spare warp per quarter does the piece ends
+  constexpr int NE = side ? Rl::kNE : W;    // epilogue (and Q-writing) warps per used quarter
   const int n_soft = R * qpc * W;           // softmax warps of each group
-  const int n_piece = R * qpc * 4;          // warps that write Q and read O
+  const int n_epi = R * qpc * NE;           // warps that write Q and finish pieces
 
   if (tid == 0) {
     for (int i = 0; i < ns; ++i) {
@@ -265,11 +287,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       mbar_init(&p_full[i], n_soft);
       mbar_init(&p_empty[i], 1);
     }
+    mbar_init(&q_full, n_epi);
+    mbar_init(&q_empty, 1);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&q_full[i], n_piece);
-      mbar_init(&q_empty[i], 1);
+      mbar_init(&o_full[i], 1);
+      mbar_init(&o_free[i], n_epi);
+      mbar_init(&ml_full[i], n_soft);
+      mbar_init(&ml_empty[i], n_epi);
     }
-    mbar_init(&o_free, n_piece);
     mbar_init(&mma_done[0], 1);
     mbar_init(&mma_done[1], 1);
     s_abort = 0;
@@ -288,12 +313,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     gpre[g + 1] = 0;
     gact[g] = 0;
   }
+  for (int i = tid; i < (p.G * p.rpg + 31) / 32; i += kAttnThreads) rowbits[i] = 0;
   if (tid == 0) gpre[0] = 0;
   __syncthreads();
   for (int r = tid; r < p.G * p.rpg; r += kAttnThreads) {
     if (!row_on(p, r)) continue;
     atomicAdd(&gpre[r / p.rpg + 1], (clamp_len(p.suffix_len[r], p.max_sp) + kPage - 1) / kPage);
     atomicOr(&gact[r / p.rpg], 1);
+    atomicOr(&rowbits[r >> 5], 1u << (r & 31));
   }
   __syncthreads();
   for (int g = tid; g < p.G; g += kAttnThreads)
@@ -474,10 +501,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       int64_t x0 = b;
       while (ok && x0 < e) {
         const int n_in = (int)(min(e, cur.start + cur.n) - x0);
-        const int qb = pc & 1;
-        if (!wait_or_abort(&q_full[qb], (uint32_t)(pc >> 1) & 1u, abort_flag)) break;
+        if (!wait_or_abort(&q_full, (uint32_t)pc & 1u, abort_flag)) break;
         tc_fence_after();
-        const uint32_t qa = tmem + kQCol + qb * (D / 2);
+        const uint32_t qa = tmem + kQCol;
         for (int k0 = 0; k0 < n_in; k0 += kGroupPages) {
           const int ng = min(kGroupPages, n_in - k0);
           const int sb = gi % kSBufs;
@@ -501,7 +527,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                              kg + (uint64_t)(((kk >> 2) * (kGroupPages * 2048) + (kk & 3) * 32) >> 4), idesc_qk,
                              kk > 0 ? 1u : 0u);
           umma_commit(&s_full[sb]);
-          if (k0 + ng == n_in) umma_commit(&q_empty[qb]);
+          if (k0 + ng == n_in) umma_commit(&q_empty);  // Q may take the next piece
           ++gi;
         }
         ++pc;
@@ -530,7 +556,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             ok = false;
             break;
           }
-          if (k0 == 0 && pc >= 1 && !wait_or_abort(&o_free, (uint32_t)(pc - 1) & 1u, abort_flag)) {
+          // a piece's O buffer is free once the piece two back has been read out
+          if (k0 == 0 && pc >= 2 && !wait_or_abort(&o_free[pc & 1], (uint32_t)((pc >> 1) - 1) & 1u, abort_flag)) {
             ok = false;
             break;
           }
@@ -538,12 +565,13 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 #pragma unroll
           for (int j = 0; j < kGroupPages; ++j) {
             if (j < ng)
-              umma_bf16_tmem_a(tmem + kOCol, tmem + kPCol + pb * 32 + j * 8,
+              umma_bf16_tmem_a(tmem + kOCol + (pc & 1) * kOStride, tmem + kPCol + pb * 32 + j * 8,
                                v_d + (uint64_t)((gs * kSlot + kVOff + j * kTile) >> 4), kIdescPV,
                                (k0 == 0 && j == 0) ? 0u : 1u);
           }
           umma_commit(&p_empty[pb]);
           umma_commit(&empty_bar[gs]);  // the slot's K and V are no longer read
+          if (k0 + ng == n_in) umma_commit(&o_full[pc & 1]);  // the piece's O is final
           ++gi;
         }
         ++pc;
@@ -561,64 +589,86 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     // the other copies' page columns, so O in its lanes sums its own pages only.
     // For nq <= 32 each page of a group is thus handled on its own SM
     // sub-partition (a warp can only reach its own lane quarter) and no warp
-    // waits for another between groups.  At the end of a job piece all four
-    // warps of every used quarter read O (a quarter of its columns each), and the
-    // copies are merged by log-sum-exp through shared memory; the next piece's Q
-    // is written before that, so its first QKs overlap the epilogue.
+    // waits for another between groups.
+    // The other 4 - W warps of each used quarter are the epilogue warps: they
+    // write the next piece's Q and, while the softmax warps go on with the next
+    // piece (into the other O buffer), read a finished piece's O, merge the
+    // copies by log-sum-exp through shared memory and write the output or the
+    // partial.  With W = 4 (no spare warps) the softmax warps do both in turn.
     const int nq = p.nq, gq = p.gq;
     const int qd = warp & 3, pj = warp >> 2;  // TMEM lane quarter; warp within the quarter
     const int cp = qd / qpc, rb = qd % qpc;   // copy; row block of the queries
-    const bool in_piece = cp < R;             // Q writes and the epilogue
-    const bool in_group = in_piece && pj < W; // the softmax of each group
-    const int jp = cp + pj * R;               // this warp's page within a group
+    const bool in_piece = cp < R;
+    const bool in_group = in_piece && pj < W;
+    const bool in_epi = in_piece && (side ? pj >= W : true);
+    const int ei = side ? pj - W : pj;        // index among the quarter's epilogue warps (< NE)
+    const int jp = cp + pj * R;               // a softmax warp's page within a group
     auto soft_sync = [&]() { asm volatile("bar.sync 1, %0;" ::"r"(n_soft * 32) : "memory"); };
-    auto piece_sync = [&]() { asm volatile("bar.sync 2, %0;" ::"r"(n_piece * 32) : "memory"); };
+    auto epi_sync = [&]() { asm volatile("bar.sync 2, %0;" ::"r"(n_epi * 32) : "memory"); };
     const int r = rb * 32 + lane;              // this thread's query
     const int rloc = r < nq ? r / gq : -2;     // its row within the group (suffix pages are per row)
     const int tlane = qd * 32 + lane;          // its TMEM lane
     const uint32_t tl = tmem + ((uint32_t)(qd * 32) << 16);
     float* rmax = reinterpret_cast<float*>(smem + L.red);  // [2][4][128] page-slot maxima
-    float* rsum = rmax + 2 * 4 * kRows;                    // [4][128] page-slot row sums
-    float* mfin = rsum + 4 * kRows;                        // [128] running max at the piece end
-    float4* stage = reinterpret_cast<float4*>(mfin + kRows);  // [<= 12][4][32] O columns of copies >= 1
+    float* rsum = rmax + 2 * 4 * kRows;                    // [2 pieces][4][128] page-slot row sums
+    float* mfin = rsum + 2 * 4 * kRows;                    // [2 pieces][128] running max at the piece end
+    float4* stage = reinterpret_cast<float4*>(mfin + 2 * kRows);  // [<= 9][4][32] O columns of copies >= 1
     const int ocols = D / W;                   // O columns rescaled by each softmax warp of a quarter
-    constexpr int kEpiCols = D / 4;            // O columns read by each warp of a quarter at the end
-    constexpr int kQCols = D / 8;              // Q columns (bf16 pairs) written by each warp of a quarter
+    constexpr int kChunks = D / 16;            // 16-column chunks of O (and 8-column chunks of Q)
     // warp-uniform bounded wait (TMEM loads and stores that follow are warp-collective)
     auto wwait = [&](uint64_t* bar, uint32_t parity, volatile int32_t* flag) {
       return __all_sync(0xffffffffu, wait_or_abort(bar, parity, flag));
     };
-    // this warp's share of its rows' queries for piece number `pn` of job `jb`
-    auto write_q = [&](const Job& jb, int pn) {
-      const int qb = pn & 1;
-      bool fine = true;
-      if (pn >= 2 && !wwait(&q_empty[qb], (uint32_t)((pn >> 1) - 1) & 1u, abort_flag)) fine = false;
-      if (fine) {
-        constexpr int kLd = kQCols / 4;  // uint4 loads: a column holds two bf16, a uint4 eight
-        uint4 qv[kLd];
-        if (r < nq) {
-          const int rr = jb.g * p.rpg + r / gq, hq = jb.h * gq + r % gq;
-          const uint4* src = reinterpret_cast<const uint4*>(p.q + ((int64_t)rr * p.Hq + hq) * D) + pj * kLd;
+    // Q of job jb: this epilogue warp's share of its rows' query columns (8-column
+    // chunks ei, ei + NE, ...), loaded first; then, if `after` is set, the wait for
+    // the last QK of the piece before, which frees the single Q buffer
+    auto write_q = [&](const Job& jb, bool after, uint32_t parity) {
+      constexpr int kMaxChunks = (kChunks + NE - 1) / NE;
+      uint4 qv[2 * kMaxChunks];
+      int n = 0;
+      const bool qrow = r < nq;
+      const uint4* src = nullptr;
+      if (qrow) {
+        const int rr = jb.g * p.rpg + r / gq, hq = jb.h * gq + r % gq;
+        src = reinterpret_cast<const uint4*>(p.q + ((int64_t)rr * p.Hq + hq) * D);
+      }
 #pragma unroll
-          for (int t = 0; t < kLd; ++t) qv[t] = __ldg(src + t);
-        } else {
-#pragma unroll
-          for (int t = 0; t < kLd; ++t) qv[t] = make_uint4(0u, 0u, 0u, 0u);
+      for (int t = 0; t < kMaxChunks; ++t) {
+        const int ch = ei + t * NE;
+        if (t * NE < kChunks && ch < kChunks) {
+          qv[2 * t] = qrow ? __ldg(src + 2 * ch) : make_uint4(0u, 0u, 0u, 0u);
+          qv[2 * t + 1] = qrow ? __ldg(src + 2 * ch + 1) : make_uint4(0u, 0u, 0u, 0u);
+          n = t + 1;
         }
-        const uint32_t qcol = kQCol + qb * (D / 2) + pj * kQCols;
+      }
+      bool fine = true;
+      if (after && !wwait(&q_empty, parity, abort_flag)) fine = false;
+      if (fine) {
+        tc_fence_after();
 #pragma unroll
-        for (int t = 0; t < kQCols / 8; ++t) {
-          const uint32_t v8[8] = {qv[2 * t].x,     qv[2 * t].y,     qv[2 * t].z,     qv[2 * t].w,
-                                  qv[2 * t + 1].x, qv[2 * t + 1].y, qv[2 * t + 1].z, qv[2 * t + 1].w};
-          tmem_st8(tl + qcol + t * 8, v8);
+        for (int t = 0; t < kMaxChunks; ++t) {
+          if (t < n) {
+            const uint32_t v8[8] = {qv[2 * t].x,     qv[2 * t].y,     qv[2 * t].z,     qv[2 * t].w,
+                                    qv[2 * t + 1].x, qv[2 * t + 1].y, qv[2 * t + 1].z, qv[2 * t + 1].w};
+            tmem_st8(tl + kQCol + (ei + t * NE) * 8, v8);
+          }
         }
         tmem_st_wait();
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&q_full[qb]);
+      if (lane == 0) mbar_arrive(&q_full);
       return fine;
     };
+
+    // P columns of pages this warp's copy does not handle must read 0 in its
+    // lanes: they are never written after this
+    if (in_group) {
+      const uint32_t zero[16] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+#pragma unroll
+      for (int c0 = 0; c0 < kPBufs * 32; c0 += 16) tmem_st16(tl + kPCol + c0, zero);
+      tmem_st_wait();
+    }
 
     // jobs with no pages at all (empty prompt and suffixes, some row active)
     for (int j = c; j < p.G * p.Hkv; j += p.C) {
@@ -633,222 +683,237 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       }
     }
 
-    // P columns of pages this warp's copy does not handle must read 0 in its
-    // lanes: they are never written after this
-    if (in_group) {
-      const uint32_t zero[16] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
-#pragma unroll
-      for (int c0 = 0; c0 < kPBufs * 32; c0 += 16) tmem_st16(tl + kPCol + c0, zero);
-      tmem_st_wait();
-    }
-
     // These warps never leave their loops early: the loop structure is the same
-    // for all of them, so every named barrier is reached even after an abort
-    // (waits then return at once and the work is skipped).
-    int gi = 0, pc = 0;
+    // for all warps of a role, so every named barrier is reached even after an
+    // abort (waits then return at once and the work is skipped).
+    int gi = 0;
     bool ok = true;
-    Job cur;
-    const int64_t x_end = in_piece ? e : b;
-    if (b < x_end) {
-      cur = job_at(p, gpre, b);
-      if (!write_q(cur, 0)) ok = false;
-    }
-    for (int64_t x0 = b; x0 < x_end;) {
-      const int n_in = (int)(min(e, cur.start + cur.n) - x0);
-      const int j = cur.g * p.Hkv + cur.h;
-      float m_used = -INFINITY, l = 0.f;  // m_used is shared by the W warps of a quarter; l is per warp
-      if (!in_group) gi += (n_in + kGroupPages - 1) / kGroupPages;
-      for (int k0 = 0; in_group && k0 < n_in; k0 += kGroupPages) {
-        const int ng = min(kGroupPages, n_in - k0);
-        const int sb = gi % kSBufs, pb = gi % kPBufs, gs = gi % ns;
-        const bool has = jp < ng;
-        int tok = 0, sel = -1;
-        if (has && ok) {
-          // this page's descriptor; the producer's write is ordered by the full barrier
-          if (wwait(&full_bar[gs], (uint32_t)(gi / ns) & 1u, abort_flag)) {
-            const uint32_t dsc = descs[gs * kGroupPages + jp];
-            tok = (int)(dsc & 0xffffu);
-            sel = (int)(int16_t)(dsc >> 16);
-          } else {
-            ok = false;
-          }
-        }
-        if (ok && !wwait(&s_full[sb], (uint32_t)(gi / kSBufs) & 1u, abort_flag)) ok = false;
-        tc_fence_after();
-        float sc[kPage];
-#pragma unroll
-        for (int t = 0; t < kPage; ++t) sc[t] = -INFINITY;
-        if (has && ok) {
-          uint32_t raw[16];
-          tmem_ld16(tl + kSCol + sb * 64 + jp * kPage, raw);
-          tmem_ld_wait();
-#pragma unroll
-          for (int t = 0; t < kPage; ++t) sc[t] = __uint_as_float(raw[t]);
-        }
-        // S is in registers: its buffer can take the group after next
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&s_empty[sb]);
-        // masks: token count of the page, and a suffix page is visible to one row only
-        const bool rowok = has && ok && rloc >= 0 && (sel < 0 || sel == rloc);
-#pragma unroll
-        for (int t = 0; t < kPage; ++t) sc[t] = (rowok && t < tok) ? sc[t] * p.scale_log2 : -INFINITY;
-        float mx = fmaxf(fmaxf(fmaxf(fmaxf(sc[0], sc[1]), fmaxf(sc[2], sc[3])), fmaxf(fmaxf(sc[4], sc[5]), fmaxf(sc[6], sc[7]))),
-                         fmaxf(fmaxf(fmaxf(sc[8], sc[9]), fmaxf(sc[10], sc[11])), fmaxf(fmaxf(sc[12], sc[13]), fmaxf(sc[14], sc[15]))));
-        if (W > 1) {
-          // the group's row max over the quarter's page slots
-          float* rm = rmax + (gi & 1) * 4 * kRows;
-          rm[pj * kRows + tlane] = mx;
-          soft_sync();
-          mx = rm[tlane];
-          for (int w = 1; w < W; ++w) mx = fmaxf(mx, rm[w * kRows + tlane]);
-        }
-        const bool need = mx > m_used + kRescaleLog2;
-        if (__any_sync(0xffffffffu, need)) {
-          const float nm = need ? mx : m_used;
-          const float f = (m_used == -INFINITY) ? 0.f : exp2f(m_used - nm);
-          const int pg = gi - 1;
-          if (k0 > 0 && ok && !wwait(&p_empty[pg % kPBufs], (uint32_t)(pg / kPBufs) & 1u, abort_flag)) ok = false;
-          if (k0 > 0 && ok) {
-            // O holds this piece's earlier groups: the last PV is done; rescale this warp's columns
-            tc_fence_after();
-#pragma unroll 1
-            for (int cc = 0; cc < ocols; cc += 16) {
-              uint32_t raw[16];
-              const uint32_t col = kOCol + pj * ocols + cc;
-              tmem_ld16(tl + col, raw);
-              tmem_ld_wait();
-#pragma unroll
-              for (int t = 0; t < 16; ++t) raw[t] = __float_as_uint(__uint_as_float(raw[t]) * f);
-              tmem_st16(tl + col, raw);
+    // the groups of one job piece (softmax warps), then the hand-off of the
+    // piece's (m, l) to the epilogue warps
+    auto run_groups = [&](const Job& cur, int n_in, int pc) {
+      const int ob = pc & 1;
+      const uint32_t ocol = kOCol + ob * kOStride;
+        float m_used = -INFINITY, l = 0.f;  // m_used is shared by the W warps of a quarter; l is per warp
+        for (int k0 = 0; k0 < n_in; k0 += kGroupPages) {
+          const int ng = min(kGroupPages, n_in - k0);
+          const int sb = gi % kSBufs, pb = gi % kPBufs, gs = gi % ns;
+          const bool has = jp < ng;
+          int tok = 0, sel = -1;
+          if (has && ok) {
+            // this page's descriptor; the producer's write is ordered by the full barrier
+            if (wwait(&full_bar[gs], (uint32_t)(gi / ns) & 1u, abort_flag)) {
+              const uint32_t dsc = descs[gs * kGroupPages + jp];
+              tok = (int)(dsc & 0xffffu);
+              sel = (int)(int16_t)(dsc >> 16);
+            } else {
+              ok = false;
             }
+          }
+          if (ok && !wwait(&s_full[sb], (uint32_t)(gi / kSBufs) & 1u, abort_flag)) ok = false;
+          tc_fence_after();
+          float sc[kPage];
+#pragma unroll
+          for (int t = 0; t < kPage; ++t) sc[t] = -INFINITY;
+          if (has && ok) {
+            uint32_t raw[16];
+            tmem_ld16(tl + kSCol + sb * 64 + jp * kPage, raw);
+            tmem_ld_wait();
+#pragma unroll
+            for (int t = 0; t < kPage; ++t) sc[t] = __uint_as_float(raw[t]);
+          }
+          // S is in registers: its buffer can take the group after next
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&s_empty[sb]);
+          // masks: token count of the page, and a suffix page is visible to one row only
+          const bool rowok = has && ok && rloc >= 0 && (sel < 0 || sel == rloc);
+#pragma unroll
+          for (int t = 0; t < kPage; ++t) sc[t] = (rowok && t < tok) ? sc[t] * p.scale_log2 : -INFINITY;
+          float mx = fmaxf(fmaxf(fmaxf(fmaxf(sc[0], sc[1]), fmaxf(sc[2], sc[3])), fmaxf(fmaxf(sc[4], sc[5]), fmaxf(sc[6], sc[7]))),
+                           fmaxf(fmaxf(fmaxf(sc[8], sc[9]), fmaxf(sc[10], sc[11])), fmaxf(fmaxf(sc[12], sc[13]), fmaxf(sc[14], sc[15]))));
+          if (W > 1) {
+            // the group's row max over the quarter's page slots
+            float* rm = rmax + (gi & 1) * 4 * kRows;
+            rm[pj * kRows + tlane] = mx;
+            soft_sync();
+            mx = rm[tlane];
+            for (int w = 1; w < W; ++w) mx = fmaxf(mx, rm[w * kRows + tlane]);
+          }
+          const bool need = mx > m_used + kRescaleLog2;
+          if (__any_sync(0xffffffffu, need)) {
+            const float nm = need ? mx : m_used;
+            const float f = (m_used == -INFINITY) ? 0.f : exp2f(m_used - nm);
+            const int pg = gi - 1;
+            if (k0 > 0 && ok && !wwait(&p_empty[pg % kPBufs], (uint32_t)(pg / kPBufs) & 1u, abort_flag)) ok = false;
+            if (k0 > 0 && ok) {
+              // O holds this piece's earlier groups: the last PV is done; rescale this warp's columns
+              tc_fence_after();
+#pragma unroll 1
+              for (int cc = 0; cc < ocols; cc += 16) {
+                uint32_t raw[16];
+                const uint32_t col = ocol + pj * ocols + cc;
+                tmem_ld16(tl + col, raw);
+                tmem_ld_wait();
+#pragma unroll
+                for (int t = 0; t < 16; ++t) raw[t] = __float_as_uint(__uint_as_float(raw[t]) * f);
+                tmem_st16(tl + col, raw);
+              }
+              tmem_st_wait();
+            }
+            l *= f;
+            m_used = nm;
+          }
+          // P = 2^(s - m) (ex2 of -inf is +0: masked tokens give 0)
+          const float ref = (m_used == -INFINITY) ? 0.f : m_used;
+          float pv[kPage];
+#pragma unroll
+          for (int t = 0; t < kPage; ++t) pv[t] = ex2_approx(sc[t] - ref);
+          uint32_t pk[kPage / 2];
+#pragma unroll
+          for (int t = 0; t < kPage; t += 2) pk[t / 2] = pack_bf16x2(pv[t], pv[t + 1]);
+          l += ((((pv[0] + pv[1]) + (pv[2] + pv[3])) + ((pv[4] + pv[5]) + (pv[6] + pv[7]))) +
+                (((pv[8] + pv[9]) + (pv[10] + pv[11])) + ((pv[12] + pv[13]) + (pv[14] + pv[15]))));
+          // the P buffer is free once the PV of the group that used it last is done
+          const int pq = gi - kPBufs;
+          if (pq >= 0 && ok && !wwait(&p_empty[pb], (uint32_t)(pq / kPBufs) & 1u, abort_flag)) ok = false;
+          if (has && ok) {
+            tc_fence_after();
+            tmem_st8(tl + kPCol + pb * 32 + jp * 8, pk);  // P of this page (the other copies' pages stay 0)
             tmem_st_wait();
           }
-          l *= f;
-          m_used = nm;
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&p_full[pb]);
+          ++gi;
         }
-        // P = 2^(s - m) (ex2 of -inf is +0: masked tokens give 0)
-        const float ref = (m_used == -INFINITY) ? 0.f : m_used;
-        float pv[kPage];
-#pragma unroll
-        for (int t = 0; t < kPage; ++t) pv[t] = ex2_approx(sc[t] - ref);
-        uint32_t pk[kPage / 2];
-#pragma unroll
-        for (int t = 0; t < kPage; t += 2) pk[t / 2] = pack_bf16x2(pv[t], pv[t + 1]);
-        l += ((((pv[0] + pv[1]) + (pv[2] + pv[3])) + ((pv[4] + pv[5]) + (pv[6] + pv[7]))) +
-              (((pv[8] + pv[9]) + (pv[10] + pv[11])) + ((pv[12] + pv[13]) + (pv[14] + pv[15]))));
-        // the P buffer is free once the PV of the group that used it last is done
-        const int pq = gi - kPBufs;
-        if (pq >= 0 && ok && !wwait(&p_empty[pb], (uint32_t)(pq / kPBufs) & 1u, abort_flag)) ok = false;
-        if (has && ok) {
-          tc_fence_after();
-          tmem_st8(tl + kPCol + pb * 32 + jp * 8, pk);  // P of this page (the other copies' pages stay 0)
-          tmem_st_wait();
-        }
-        tc_fence_before();
+        // hand the piece's (m, l) to the epilogue warps (slot reused two pieces on)
+        if (pc >= 2 && ok && !wwait(&ml_empty[ob], (uint32_t)((pc >> 1) - 1) & 1u, abort_flag)) ok = false;
+        rsum[(ob * 4 + pj) * kRows + tlane] = l;
+        if (pj == 0) mfin[ob * kRows + tlane] = m_used;
         __syncwarp();
-        if (lane == 0) mbar_arrive(&p_full[pb]);
-        ++gi;
-      }
-      // ---- the next piece's Q goes in first, so that its QKs overlap this epilogue ----
-      Job nxt = cur;
-      const bool more = x0 + n_in < e;
-      if (more) {
-        nxt = next_job(p, gpre, cur);
-        if (!write_q(nxt, pc + 1)) ok = false;
-      }
-      // ---- end of the piece: O is final once the last group's PV completes ----
-      const int lg = gi - 1;
-      if (ok && !wwait(&p_empty[lg % kPBufs], (uint32_t)(lg / kPBufs) & 1u, abort_flag)) ok = false;
-      tc_fence_after();
-      if (in_group) {
-        rsum[pj * kRows + tlane] = l;
-        if (pj == 0) mfin[tlane] = m_used;
-      }
-      piece_sync();
-      // the copies' running maxima and row sums -> the piece's max M and sum L;
-      // copy c's O is weighted by 2^(m_c - M)
-      float M = -INFINITY, Ls = 0.f;
-      for (int c2 = 0; c2 < R; ++c2) M = fmaxf(M, mfin[(c2 * qpc + rb) * 32 + lane]);
-      for (int c2 = 0; c2 < R; ++c2) {
-        const int ln = (c2 * qpc + rb) * 32 + lane;
-        float Lc = 0.f;
-        for (int w = 0; w < W; ++w) Lc += rsum[w * kRows + ln];
-        if (mfin[ln] != -INFINITY) Ls += exp2f(mfin[ln] - M) * Lc;
-      }
-      const float wself = mfin[tlane] == -INFINITY ? 0.f : exp2f(mfin[tlane] - M);
-      const int first = cta_of(cur.start, T, Ceff), last = cta_of(cur.start + cur.n - 1, T, Ceff);
-      const bool mine_row = r < nq && cp == 0;
-      const int rr = r < nq ? cur.g * p.rpg + r / gq : 0, hq = r < nq ? cur.h * gq + r % gq : 0;
-      const bool write_row = mine_row && row_on(p, rr);
-      const int64_t s_idx = (int64_t)c + j;
-      const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-      // after an abort the piece's outputs are not written (the status word says so)
-      const bool out_ok = __all_sync(0xffffffffu, ok && !*abort_flag);
-      // O, 16 columns per round; copies >= 1 pass theirs to copy 0 through shared memory
-      const int my_stage = ((cp - 1) * qpc + rb) * 4 + pj;  // (for copies >= 1)
-#pragma unroll 1
-      for (int cc = 0; cc < kEpiCols; cc += 16) {
-        const int col = pj * kEpiCols + cc;
-        float o[16];
-        if (out_ok) {
-          uint32_t raw[16];
-          tmem_ld16(tl + kOCol + col, raw);
-          tmem_ld_wait();
-#pragma unroll
-          for (int t = 0; t < 16; ++t) o[t] = __uint_as_float(raw[t]) * wself;
+        if (lane == 0) mbar_arrive(&ml_full[ob]);
+          };
+    // the next piece's Q, then this piece's end (epilogue warps)
+    auto run_epilogue = [&](const Job& cur, int pc, bool more, const Job& nxt) {
+      const int j = cur.g * p.Hkv + cur.h;
+      const int ob = pc & 1;
+      const uint32_t ocol = kOCol + ob * kOStride;
+        // ---- the next piece's Q, once this piece's last QK is done ----
+        if (more && !write_q(nxt, true, (uint32_t)pc & 1u)) ok = false;
+        // ---- this piece's epilogue: O is final once its last PV completes ----
+        const int first = cta_of(cur.start, T, Ceff), last = cta_of(cur.start + cur.n - 1, T, Ceff);
+        const int rr = r < nq ? cur.g * p.rpg + r / gq : 0, hq = r < nq ? cur.h * gq + r % gq : 0;
+        const bool mine_row = r < nq && cp == 0;
+        const bool write_row = mine_row && ((rowbits[rr >> 5] >> (rr & 31)) & 1u);
+        if (ok && !wwait(&o_full[ob], (uint32_t)(pc >> 1) & 1u, abort_flag)) ok = false;
+        if (ok && !wwait(&ml_full[ob], (uint32_t)(pc >> 1) & 1u, abort_flag)) ok = false;
+        tc_fence_after();
+        // the copies' running maxima and row sums -> the piece's max M and sum L;
+        // copy c's O is weighted by 2^(m_c - M)
+        float M = -INFINITY, Ls = 0.f;
+        for (int c2 = 0; c2 < R; ++c2) M = fmaxf(M, mfin[ob * kRows + (c2 * qpc + rb) * 32 + lane]);
+        for (int c2 = 0; c2 < R; ++c2) {
+          const int ln = (c2 * qpc + rb) * 32 + lane;
+          float Lc = 0.f;
+          for (int w = 0; w < W; ++w) Lc += rsum[(ob * 4 + w) * kRows + ln];
+          const float mc = mfin[ob * kRows + ln];
+          if (mc != -INFINITY) Ls += exp2f(mc - M) * Lc;
         }
-        if (R > 1) {
-          if (cc > 0) piece_sync();  // the previous round's staging has been read
-          if (cp > 0 && out_ok) {
-#pragma unroll
-            for (int t = 0; t < 4; ++t)
-              stage[(my_stage * 4 + t) * 32 + lane] = make_float4(o[4 * t], o[4 * t + 1], o[4 * t + 2], o[4 * t + 3]);
-          }
-          piece_sync();
-          if (cp == 0 && out_ok) {
+        const float mself = mfin[ob * kRows + tlane];
+        const float wself = mself == -INFINITY ? 0.f : exp2f(mself - M);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&ml_empty[ob]);  // the (m, l) slot has been read
+        const int64_t s_idx = (int64_t)c + j;
+        const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+        // after an abort the piece's outputs are not written (the status word says so)
+        const bool out_ok = __all_sync(0xffffffffu, ok && !*abort_flag);
+        // O in 16-column chunks: epilogue warp ei of a quarter takes chunks ei,
+        // ei + NE, ...; copies >= 1 pass theirs to copy 0 through shared memory
+        constexpr int rounds = (kChunks + NE - 1) / NE;
+        const int my_stage = ((cp - 1) * qpc + rb) * NE + ei;  // (for copies >= 1)
 #pragma unroll 1
-            for (int c2 = 1; c2 < R; ++c2) {
-              const float4* src4 = stage + ((((c2 - 1) * qpc + rb) * 4 + pj) * 4) * 32 + lane;
+        for (int rd = 0; rd < rounds; ++rd) {
+          const int ch = ei + rd * NE;
+          const bool has = ch < kChunks && out_ok;
+          const int col = ch * 16;
+          float o[16];
+          if (has) {
+            uint32_t raw[16];
+            tmem_ld16(tl + ocol + col, raw);
+            tmem_ld_wait();
 #pragma unroll
-              for (int t = 0; t < 4; ++t) {
-                const float4 v = src4[t * 32];
-                o[4 * t] += v.x;
-                o[4 * t + 1] += v.y;
-                o[4 * t + 2] += v.z;
-                o[4 * t + 3] += v.w;
+            for (int t = 0; t < 16; ++t) o[t] = __uint_as_float(raw[t]) * wself;
+          }
+          if (R > 1) {
+            if (rd > 0) epi_sync();  // the previous round's staging has been read
+            if (cp > 0 && has) {
+#pragma unroll
+              for (int t = 0; t < 4; ++t)
+                stage[(my_stage * 4 + t) * 32 + lane] = make_float4(o[4 * t], o[4 * t + 1], o[4 * t + 2], o[4 * t + 3]);
+            }
+            epi_sync();
+            if (cp == 0 && has) {
+#pragma unroll 1
+              for (int c2 = 1; c2 < R; ++c2) {
+                const float4* src4 = stage + ((((c2 - 1) * qpc + rb) * NE + ei) * 4) * 32 + lane;
+#pragma unroll
+                for (int t = 0; t < 4; ++t) {
+                  const float4 v = src4[t * 32];
+                  o[4 * t] += v.x;
+                  o[4 * t + 1] += v.y;
+                  o[4 * t + 2] += v.z;
+                  o[4 * t + 3] += v.w;
+                }
               }
             }
           }
-        }
-        if (!out_ok) continue;
-        if (first == last) {
-          if (write_row) {
-            uint4* dst = reinterpret_cast<uint4*>(p.out + ((int64_t)rr * p.Hq + hq) * D + col);
-            dst[0] = make_uint4(pack_bf16x2(o[0] * inv, o[1] * inv), pack_bf16x2(o[2] * inv, o[3] * inv),
-                                pack_bf16x2(o[4] * inv, o[5] * inv), pack_bf16x2(o[6] * inv, o[7] * inv));
-            dst[1] = make_uint4(pack_bf16x2(o[8] * inv, o[9] * inv), pack_bf16x2(o[10] * inv, o[11] * inv),
-                                pack_bf16x2(o[12] * inv, o[13] * inv), pack_bf16x2(o[14] * inv, o[15] * inv));
-          }
-        } else if (mine_row) {
-          float4* dst = reinterpret_cast<float4*>(p.slot_o + (s_idx * nq + r) * D + col);
+          if (!has) continue;
+          if (first == last) {
+            if (write_row) {
+              uint4* dst = reinterpret_cast<uint4*>(p.out + ((int64_t)rr * p.Hq + hq) * D + col);
+              dst[0] = make_uint4(pack_bf16x2(o[0] * inv, o[1] * inv), pack_bf16x2(o[2] * inv, o[3] * inv),
+                                  pack_bf16x2(o[4] * inv, o[5] * inv), pack_bf16x2(o[6] * inv, o[7] * inv));
+              dst[1] = make_uint4(pack_bf16x2(o[8] * inv, o[9] * inv), pack_bf16x2(o[10] * inv, o[11] * inv),
+                                  pack_bf16x2(o[12] * inv, o[13] * inv), pack_bf16x2(o[14] * inv, o[15] * inv));
+            }
+          } else if (mine_row) {
+            float4* dst = reinterpret_cast<float4*>(p.slot_o + (s_idx * nq + r) * D + col);
 #pragma unroll
-          for (int t = 0; t < 4; ++t) dst[t] = make_float4(o[4 * t], o[4 * t + 1], o[4 * t + 2], o[4 * t + 3]);
+            for (int t = 0; t < 4; ++t) dst[t] = make_float4(o[4 * t], o[4 * t + 1], o[4 * t + 2], o[4 * t + 3]);
+          }
         }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&o_free[ob]);  // this O buffer may take the piece after next
+        if (first == last) {
+          if (out_ok && ei == 0 && write_row && p.lse)
+            p.lse[(int64_t)rr * p.Hq + hq] = Ls > 0.f ? (M + log2f(Ls)) * kLn2 : -INFINITY;
+        } else if (out_ok && ei == 0 && mine_row) {
+          p.slot_ml[s_idx * nq + r] = make_float2(M, Ls);  // the merge kernel finishes the job
+        }
+        if (R > 1) epi_sync();  // the staging buffer is reused at the next piece
+          };
+    const int64_t x_end = in_piece ? e : b;
+    if (b < x_end) {
+      Job cur = job_at(p, gpre, b);
+      if (in_epi && !write_q(cur, false, 0u)) ok = false;
+      int pc = 0;
+      for (int64_t x0 = b; x0 < x_end; ++pc) {
+        const int n_in = (int)(min(e, cur.start + cur.n) - x0);
+        const bool more = x0 + n_in < e;
+        const Job nxt = more ? next_job(p, gpre, cur) : cur;
+        if (side) {
+          // one role per warp: the softmax warps run ahead into the next piece
+          // while the epilogue warps finish this one
+          if (in_group) run_groups(cur, n_in, pc);
+          else run_epilogue(cur, pc, more, nxt);
+        } else {
+          run_groups(cur, n_in, pc);
+          run_epilogue(cur, pc, more, nxt);
+        }
+        x0 += n_in;
+        cur = nxt;
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&o_free);
-      if (first == last) {
-        if (out_ok && pj == 0 && write_row && p.lse)
-          p.lse[(int64_t)rr * p.Hq + hq] = Ls > 0.f ? (M + log2f(Ls)) * kLn2 : -INFINITY;
-      } else if (out_ok && pj == 0 && mine_row) {
-        p.slot_ml[s_idx * nq + r] = make_float2(M, Ls);  // the merge kernel finishes the job
-      }
-      piece_sync();  // the exchange buffers are reused at the next piece
-      ++pc;
-      x0 += n_in;
-      cur = nxt;
     }
   }
   tc_fence_before();
@@ -1046,7 +1111,9 @@ int make_plan(const rgd_attn_shape* s, Plan* pl) {
   // its PV, which is issued after the next group's QK.
   pl->nslots = kMaxSlots;
   for (;;) {
-    pl->smem = s->head_dim == 128 ? smem_layout<128>(pl->nslots, s->num_groups) : smem_layout<64>(pl->nslots, s->num_groups);
+    const int R = s->num_groups * s->rows_per_group;
+    pl->smem = s->head_dim == 128 ? smem_layout<128>(pl->nslots, s->num_groups, R)
+                                  : smem_layout<64>(pl->nslots, s->num_groups, R);
     if (pl->smem.total <= kSmemLimit) break;
     if (pl->nslots <= 3)
       return set_error(RGD_ERR_UNSUPPORTED, "shape needs more shared memory than an SM has (too many groups?)");
@@ -1078,6 +1145,24 @@ extern "C" size_t rgd_prefix_decode_attn_workspace_size(const rgd_attn_shape* sh
   if (make_plan(shape, &pl) != RGD_OK) return 0;
   return pl.total;
 }
+
+namespace rgd {
+namespace {
+
+// The attention kernel for one (head dim, copy count), then the split-job merge.
+template <int D, int R>
+int launch_attn(const CUtensorMap& tmK, const CUtensorMap& tmV, const AttnParams& p, const Plan& pl,
+                cudaStream_t st) {
+  static bool done = false;
+  if (int rc = ensure_smem(attn_tc_kernel<D, R>, kSmemLimit, &done)) return rc;
+  attn_tc_kernel<D, R><<<pl.C, Roles<R>::kThreads, pl.smem.total, st>>>(tmK, tmV, p);
+  if (cudaError_t e = cudaGetLastError(); e != cudaSuccess) return cuda_error(e, "attention launch");
+  if (cudaError_t e = launch_merge<D>(p, pl.J, st); e != cudaSuccess) return cuda_error(e, "merge launch");
+  return RGD_OK;
+}
+
+}  // namespace
+}  // namespace rgd
 
 extern "C" int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf16* q, const rgd_bf16* k_pages,
                                       const rgd_bf16* v_pages, const int32_t* prompt_block_table,
@@ -1131,19 +1216,19 @@ extern "C" int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf1
   p.scale_log2 = softmax_scale * kLog2e;
 
   cudaStream_t st = (cudaStream_t)stream;
+  const int qpc = (pl.nq + 31) / 32;
+  const int R = qpc == 1 ? 4 : qpc == 2 ? 2 : 1;  // copies of the queries in the TMEM lanes
+  int rc = RGD_OK;
   if (s.head_dim == 128) {
-    static bool done = false;
-    if (int rc = ensure_smem(attn_tc_kernel<128>, kSmemLimit, &done)) return rc;
-    attn_tc_kernel<128><<<pl.C, kAttnThreads, pl.smem.total, st>>>(tmK, tmV, p);
-    if (cudaError_t e = cudaGetLastError(); e != cudaSuccess) return cuda_error(e, "attention launch");
-    if (cudaError_t e = launch_merge<128>(p, pl.J, st); e != cudaSuccess) return cuda_error(e, "merge launch");
+    rc = R == 4 ? launch_attn<128, 4>(tmK, tmV, p, pl, st)
+       : R == 2 ? launch_attn<128, 2>(tmK, tmV, p, pl, st)
+                : launch_attn<128, 1>(tmK, tmV, p, pl, st);
   } else {
-    static bool done = false;
-    if (int rc = ensure_smem(attn_tc_kernel<64>, kSmemLimit, &done)) return rc;
-    attn_tc_kernel<64><<<pl.C, kAttnThreads, pl.smem.total, st>>>(tmK, tmV, p);
-    if (cudaError_t e = cudaGetLastError(); e != cudaSuccess) return cuda_error(e, "attention launch");
-    if (cudaError_t e = launch_merge<64>(p, pl.J, st); e != cudaSuccess) return cuda_error(e, "merge launch");
+    rc = R == 4 ? launch_attn<64, 4>(tmK, tmV, p, pl, st)
+       : R == 2 ? launch_attn<64, 2>(tmK, tmV, p, pl, st)
+                : launch_attn<64, 1>(tmK, tmV, p, pl, st);
   }
+  if (rc) return rc;
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? RGD_OK : cuda_error(e, "attention launch");
 }
