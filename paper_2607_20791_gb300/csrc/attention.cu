@@ -78,7 +78,7 @@ struct Roles {
 constexpr int kMaxAttnWarps = Roles<1>::kThreads / 32;
 constexpr int kGroupPages = 4;                // pages per S / P buffer (64 tokens)
 constexpr int kMaxSlots = 8;                  // ring slots, one page group each
-constexpr int kSBufs = 2;                     // S buffers in TMEM (freed once the softmax has read them)
+constexpr int kSBufs = 1;                     // S buffers in TMEM (freed once the softmax has read them)
 constexpr int kPBufs = 2;                     // P buffers in TMEM (freed once their PV is done)
 constexpr int kRows = 128;                    // MMA M: query rows per job
 constexpr int kMaxQueries = kRows;            // rows_per_group * Hq / Hkv
@@ -86,8 +86,9 @@ constexpr int kTmemCols = 512;
 constexpr int kOCol = 0;                      // O: two buffers (alternate job pieces) of D columns
 constexpr int kOStride = 128;
 constexpr int kSCol = 2 * kOStride;           // S buffers: 64 fp32 columns each (4 pages x 16 tokens)
-constexpr int kPCol = kSCol + kSBufs * 64;    // P buffers: 32 columns each (4 pages x 16 bf16)
-constexpr int kQCol = kPCol + kPBufs * 32;    // Q: D/2 columns (two bf16 per column)
+constexpr int kPCol = kSCol + kSBufs * 64;    // P buffers: 32 columns each (4 pages x 16 bf16), high parts
+constexpr int kPLoCol = kPCol + kPBufs * 32;  // the matching bf16 residuals P - bf16(P)
+constexpr int kQCol = kPLoCol + kPBufs * 32;  // Q: D/2 columns (two bf16 per column)
 static_assert(kQCol + 64 <= 512, "TMEM columns");
 // V as the MN-major B operand of PV: the two 64-column halves of a page tile are
 // MN-direction swizzle atoms 2048 B apart, the two 8-token groups K-direction
@@ -562,12 +563,15 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
             break;
           }
           tc_fence_after();
+          // P = bf16 high part + bf16 residual: two MMAs per page keep ~16 bits of P
 #pragma unroll
           for (int j = 0; j < kGroupPages; ++j) {
-            if (j < ng)
-              umma_bf16_tmem_a(tmem + kOCol + (pc & 1) * kOStride, tmem + kPCol + pb * 32 + j * 8,
-                               v_d + (uint64_t)((gs * kSlot + kVOff + j * kTile) >> 4), kIdescPV,
-                               (k0 == 0 && j == 0) ? 0u : 1u);
+            if (j < ng) {
+              const uint64_t vd = v_d + (uint64_t)((gs * kSlot + kVOff + j * kTile) >> 4);
+              const uint32_t od = tmem + kOCol + (pc & 1) * kOStride;
+              umma_bf16_tmem_a(od, tmem + kPCol + pb * 32 + j * 8, vd, kIdescPV, (k0 == 0 && j == 0) ? 0u : 1u);
+              umma_bf16_tmem_a(od, tmem + kPLoCol + pb * 32 + j * 8, vd, kIdescPV, 1u);
+            }
           }
           umma_commit(&p_empty[pb]);
           umma_commit(&empty_bar[gs]);  // the slot's K and V are no longer read
@@ -666,7 +670,7 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
     if (in_group) {
       const uint32_t zero[16] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
 #pragma unroll
-      for (int c0 = 0; c0 < kPBufs * 32; c0 += 16) tmem_st16(tl + kPCol + c0, zero);
+      for (int c0 = 0; c0 < 2 * kPBufs * 32; c0 += 16) tmem_st16(tl + kPCol + c0, zero);  // high and residual
       tmem_st_wait();
     }
 
@@ -768,9 +772,14 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
           float pv[kPage];
 #pragma unroll
           for (int t = 0; t < kPage; ++t) pv[t] = ex2_approx(sc[t] - ref);
-          uint32_t pk[kPage / 2];
+          // P in bf16 as a high part and the residual (P - high), each bf16
+          uint32_t pk[kPage / 2], pl[kPage / 2];
 #pragma unroll
-          for (int t = 0; t < kPage; t += 2) pk[t / 2] = pack_bf16x2(pv[t], pv[t + 1]);
+          for (int t = 0; t < kPage; t += 2) {
+            pk[t / 2] = pack_bf16x2(pv[t], pv[t + 1]);
+            const float h0 = __uint_as_float(pk[t / 2] << 16), h1 = __uint_as_float(pk[t / 2] & 0xffff0000u);
+            pl[t / 2] = pack_bf16x2(pv[t] - h0, pv[t + 1] - h1);
+          }
           l += ((((pv[0] + pv[1]) + (pv[2] + pv[3])) + ((pv[4] + pv[5]) + (pv[6] + pv[7]))) +
                 (((pv[8] + pv[9]) + (pv[10] + pv[11])) + ((pv[12] + pv[13]) + (pv[14] + pv[15]))));
           // the P buffer is free once the PV of the group that used it last is done
@@ -779,6 +788,7 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
           if (has && ok) {
             tc_fence_after();
             tmem_st8(tl + kPCol + pb * 32 + jp * 8, pk);  // P of this page (the other copies' pages stay 0)
+            tmem_st8(tl + kPLoCol + pb * 32 + jp * 8, pl);
             tmem_st_wait();
           }
           tc_fence_before();

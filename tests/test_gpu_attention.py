@@ -104,6 +104,18 @@ def test_query_tiles_per_group(gpu_lib):
         _check(case, _run(case, num_ctas=5))
 
 
+@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("rpg,Hq,Hkv,ctas", [(11, 24, 8, 0), (5, 64, 8, 3), (8, 64, 8, 1), (12, 64, 8, 7)])
+def test_query_copy_counts(gpu_lib, D, rpg, Hq, Hkv, ctas):
+    # queries per kv head 33, 40, 64 (two copies of the queries in the tensor
+    # memory lanes) and 96 (one copy over three lane quarters), with jobs split
+    # over blocks and whole jobs in one block
+    G = 3
+    slens = [(7 * i) % 70 for i in range(G * rpg)]
+    case = workloads.make_attn_case("copies", G, rpg, Hq, Hkv, D, [0, 45, 230], slens, seed=rpg + D)
+    _check(case, _run(case, num_ctas=ctas))
+
+
 def test_masked_rows_and_groups(gpu_lib):
     active = np.array([1, 0, 1, 0, 0, 0, 0, 1, 1], np.uint8)  # group 1 fully masked
     case = workloads.make_attn_case("mask", 3, 3, 8, 2, 128, [50, 70, 90], [3, 4, 5, 6, 7, 8, 0, 0, 20],
