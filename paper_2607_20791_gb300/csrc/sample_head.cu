@@ -131,6 +131,8 @@ struct Shared {
   float red_s[kHeadWarps];
   int32_t red_c[kHeadWarps];
   float stripe_sum[kHeadWarps][kMaxStripes];
+  float stripe_max[kHeadWarps][kMaxStripes];
+  uint8_t stripe_list[kHeadWarps][kMaxStripes];  // pass 2: the stripes a warp re-reads
   // published to the cluster
   float cta_max;
   int32_t cta_arg;
@@ -155,10 +157,15 @@ struct KSum {
   __device__ __forceinline__ float value() const { return s - c; }
 };
 
-// The kept weight of logit l (0 when below the cutoff); the same fp32 steps
-// everywhere, so pass 2 and the draw agree bit for bit.
-__device__ __forceinline__ float kept_weight(float l, float cut, float M, float temp) {
-  return l >= cut ? expf(__fdiv_rn(__fsub_rn(l, M), temp)) : 0.f;
+// The kept weight exp((l - M) / T) = 2^((l - M) log2(e) / T) of logit l, 0 below
+// the cutoff; kexp = log2(e) / T per row.  The same fp32 steps everywhere, so
+// pass 2 and the draw agree bit for bit.  Against exact weights the relative
+// error is the factor's rounding times the exponent plus the 2^x unit's 2 ulp:
+// a few 1e-7 for the weights that carry the mass (exponents near 0), inside the
+// 1e-6 of Z within which a draw counts as a boundary case; weights below 2^-126
+// flush to 0.
+__device__ __forceinline__ float kept_weight(float l, float cut, float M, float kexp) {
+  return l >= cut ? ex2_approx(__fsub_rn(l, M) * kexp) : 0.f;
 }
 
 template <typename T, bool kAligned>
@@ -210,14 +217,20 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
     for (int b = 0; b < kBatch; ++b) {
       if (s0 + b >= spw) break;
       const int32_t base = (int32_t)elem(warp, s0 + b, 0);
+      float sm = -INFINITY;
 #pragma unroll
       for (int k = 0; k < kN; ++k) {
         const float v = V::get(w[b], k);
+        sm = fmaxf(sm, v);
         if (v > bv) {  // indices only grow along a lane: strict > keeps the lowest
           bv = v;
           bi = base + k;
         }
       }
+      // the stripe's maximum: pass 2 skips stripes that cannot hold a kept token
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) sm = fmaxf(sm, __shfl_xor_sync(0xffffffffu, sm, o));
+      if (lane == 0) sh.stripe_max[warp][s0 + b] = sm;
     }
   }
 #pragma unroll
@@ -297,18 +310,34 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
 
   // ---- pass 2: kept weights; the sum of every stripe and of every warp -------
   const float cut = sh.cut;
+  const float kexp = 1.4426950408889634f / temp;
   uint8_t* mask = p.kept_mask ? p.kept_mask + (int64_t)row * p.vocab : nullptr;
   KSum wsum;  // identical in every lane
   int32_t cnt = 0;
-  for (int s0 = 0; s0 < spw; s0 += kBatch) {
+  // Only stripes whose maximum reaches the cutoff can hold a kept token: the
+  // warp lists them (in index order) and re-reads just those; the others' sums
+  // are 0.  With a kept mask requested every stripe is visited.
+  for (int st = lane; st < spw; st += 32) sh.stripe_sum[warp][st] = 0.f;
+  int nlist = 0;
+  for (int s0 = 0; s0 < spw; s0 += 32) {
+    const bool hit = s0 + lane < spw && (mask != nullptr || sh.stripe_max[warp][s0 + lane] >= cut);
+    const uint32_t bal = __ballot_sync(0xffffffffu, hit);
+    if (hit) sh.stripe_list[warp][nlist + __popc(bal & ((1u << lane) - 1u))] = (uint8_t)(s0 + lane);
+    nlist += __popc(bal);
+  }
+  __syncwarp();
+  for (int i0 = 0; i0 < nlist; i0 += kBatch) {
     uint4 w[kBatch];
-#pragma unroll
-    for (int b = 0; b < kBatch; ++b)
-      if (s0 + b < spw) w[b] = load_vec<T, kAligned>(rowp, elem(warp, s0 + b, 0), p.vocab, drop_pol);
+    int sidx[kBatch];
 #pragma unroll
     for (int b = 0; b < kBatch; ++b) {
-      if (s0 + b >= spw) break;
-      const int32_t base = (int32_t)elem(warp, s0 + b, 0);
+      sidx[b] = i0 + b < nlist ? sh.stripe_list[warp][i0 + b] : 0;
+      if (i0 + b < nlist) w[b] = load_vec<T, kAligned>(rowp, elem(warp, sidx[b], 0), p.vocab, drop_pol);
+    }
+#pragma unroll
+    for (int b = 0; b < kBatch; ++b) {
+      if (i0 + b >= nlist) break;
+      const int32_t base = (int32_t)elem(warp, sidx[b], 0);
       // the lane's kept elements as a bit mask (the padding past the vocabulary reads -inf)
       uint32_t km = 0;
 #pragma unroll
@@ -320,7 +349,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
       while (km) {
         const int k = __ffs(km) - 1;
         km &= km - 1;
-        ls += expf(__fdiv_rn(__fsub_rn(V::get(w[b], k), M), temp));
+        ls += ex2_approx(__fsub_rn(V::get(w[b], k), M) * kexp);
       }
       if (mask) {
 #pragma unroll
@@ -330,7 +359,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
       float S = ls;
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) S += __shfl_xor_sync(0xffffffffu, S, o);
-      if (lane == 0) sh.stripe_sum[warp][s0 + b] = S;
+      if (lane == 0) sh.stripe_sum[warp][sidx[b]] = S;
       wsum.add(S);
     }
   }
@@ -365,80 +394,85 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
   if (warp == 0) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) cc += __shfl_xor_sync(0xffffffffu, cc, o);
-    // every lane forms the same prefix sums over the CTAs in rank order
-    KSum pre;
-    float lo = 0.f, hi = 0.f, mine = 0.f;
-    int last_nz = -1;
-    for (int r = 0; r < kClusterCtas; ++r) {
-      const float v = __shfl_sync(0xffffffffu, cs, r);
-      if (r == rank) {
-        lo = pre.value();
-        mine = v;
+    // inclusive prefix sums in double over the lanes (a handful of values per row)
+    auto scan = [&](double v) {
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const double t = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += t;
       }
-      pre.add(v);
-      if (r == rank) hi = pre.value();
-      if (v > 0.f) last_nz = r;
-    }
-    const float target = __shfl_sync(0xffffffffu, u, 0) * pre.value();
+      return v;
+    };
+    // the CTAs' sums in rank order: CTA r owns [incl(r-1), incl(r)), which tile [0, Z)
+    const double ci = scan((double)cs);
+    double ce = __shfl_up_sync(0xffffffffu, ci, 1);  // every lane takes part in the shuffle
+    if (lane == 0) ce = 0.0;
+    const double Z = __shfl_sync(0xffffffffu, ci, kClusterCtas - 1);
+    const double target = (double)__shfl_sync(0xffffffffu, u, 0) * Z;
+    const double lo = __shfl_sync(0xffffffffu, ce, rank), hi = __shfl_sync(0xffffffffu, ci, rank);
+    const uint32_t nzc = __ballot_sync(0xffffffffu, lane < kClusterCtas && cs > 0.f);
+    const float mine = __shfl_sync(0xffffffffu, cs, rank);
     if (lane == 0 && rank == 0 && p.kept_count) p.kept_count[row] = cc;
-    if (mine > 0.f && lo <= target && (target < hi || rank == last_nz)) {
-      // the warp, then the stripe, whose range holds the target (the last nonzero
-      // one if rounding leaves the target past every range)
-      KSum wp;
-      wp.add(lo);
-      int cw = -1;
-      float wbase = 0.f;
-      for (int w = 0; w < kHeadWarps; ++w) {
-        const float v = sh.red_s[w];
-        const float before = wp.value();
-        wp.add(v);
-        if (v > 0.f) {
-          cw = w;
-          wbase = before;
-          if (target < wp.value()) break;
+    if (mine > 0.f && lo <= target && (target < hi || rank == 31 - __clz(nzc))) {
+      // the warp whose range holds the target (the last nonzero one if rounding
+      // leaves the target past every range), then its stripe, the same way
+      const float wsv = lane < kHeadWarps ? sh.red_s[lane] : 0.f;
+      const double wi = lo + scan((double)wsv);
+      const uint32_t whit = __ballot_sync(0xffffffffu, wsv > 0.f && target < wi);
+      const uint32_t wnz = __ballot_sync(0xffffffffu, wsv > 0.f);
+      int cw = whit ? __ffs(whit) - 1 : (wnz ? 31 - __clz(wnz) : 0);
+      const double wbase = __shfl_sync(0xffffffffu, wi, cw) - (double)__shfl_sync(0xffffffffu, wsv, cw);
+      int cst = -1, fb = -1;
+      double sbase = wbase, run = wbase, fb_base = wbase;
+      for (int s0 = 0; s0 < spw && cst < 0; s0 += 32) {
+        const float sv = s0 + lane < spw ? sh.stripe_sum[cw][s0 + lane] : 0.f;
+        const double si = run + scan((double)sv);
+        const uint32_t shit = __ballot_sync(0xffffffffu, sv > 0.f && target < si);
+        const uint32_t snz = __ballot_sync(0xffffffffu, sv > 0.f);
+        const bool last = s0 + 32 >= spw;
+        if (shit || (last && snz)) {
+          const int L = shit ? __ffs(shit) - 1 : 31 - __clz(snz);
+          cst = s0 + L;
+          sbase = __shfl_sync(0xffffffffu, si, L) - (double)__shfl_sync(0xffffffffu, sv, L);
+        } else if (snz) {
+          // remember this round's last nonzero stripe in case rounding runs past the end
+          const int L = 31 - __clz(snz);
+          fb = s0 + L;
+          fb_base = __shfl_sync(0xffffffffu, si, L) - (double)__shfl_sync(0xffffffffu, sv, L);
         }
-      }
-      KSum sp;
-      sp.add(wbase);
-      int cst = -1;
-      float sbase = 0.f;
-      for (int st = 0; st < spw; ++st) {
-        const float v = sh.stripe_sum[cw][st];
-        const float before = sp.value();
-        sp.add(v);
-        if (v > 0.f) {
-          cst = st;
-          sbase = before;
-          if (target < sp.value()) break;
-        }
+        run = __shfl_sync(0xffffffffu, si, 31);
       }
       // (a warp or stripe is always found: a range with a nonzero sum has a
       // nonzero part; the guard only keeps a broken invariant from reading out of range)
-      if (cw < 0 || cst < 0) cw = cst = 0;
+      if (cst < 0 && fb >= 0) {
+        cst = fb;
+        sbase = fb_base;
+      }
+      if (cst < 0) cw = cst = 0;
       // the stripe's lanes: the same weights as pass 2, an inclusive scan in index order
       const uint4 w = load_vec<T, kAligned>(rowp, elem(cw, cst, 0), p.vocab, drop_pol);
       float ls = 0.f;
 #pragma unroll
-      for (int k = 0; k < kN; ++k) ls += kept_weight(V::get(w, k), cut, M, temp);
+      for (int k = 0; k < kN; ++k) ls += kept_weight(V::get(w, k), cut, M, kexp);
       float incl = ls;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
         const float v = __shfl_up_sync(0xffffffffu, incl, o);
         if (lane >= o) incl += v;
       }
-      const uint32_t over = __ballot_sync(0xffffffffu, ls > 0.f && sbase + incl > target);
+      const uint32_t over = __ballot_sync(0xffffffffu, ls > 0.f && sbase + (double)incl > target);
       const uint32_t kept_lanes = __ballot_sync(0xffffffffu, ls > 0.f);
       const int L = over ? __ffs(over) - 1 : (kept_lanes ? 31 - __clz(kept_lanes) : 0);
       int32_t tok = -1;
       if (lane == L) {
-        float r2 = sbase + (incl - ls);
+        double r2 = sbase + (double)(incl - ls);
         int32_t lk = -1;
 #pragma unroll
         for (int k = 0; k < kN; ++k) {
-          const float wk = kept_weight(V::get(w, k), cut, M, temp);
+          const float wk = kept_weight(V::get(w, k), cut, M, kexp);
           if (wk > 0.f) {
             lk = (int32_t)elem(cw, cst, k);
-            r2 += wk;
+            r2 += (double)wk;
             if (r2 > target && tok < 0) tok = lk;
           }
         }
