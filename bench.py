@@ -296,7 +296,7 @@ def run_ours(args):
                 head_gate_call()
             graphs = [g_attn, g_hg]
         torch.cuda.synchronize()
-    launches_per_step = 5  # attention, split-job merge, sample head, gate-state reset, gate
+    launches_per_step = 4  # attention (split jobs merged inside), sample head, gate-state reset, gate
 
     def one_step():
         """Runs one timed step; returns (step, attention, head + gate) in ms."""
@@ -402,14 +402,14 @@ def run_ours(args):
             "config": {"workload": WORKLOAD, "rows_per_step": rows_per_step, "groups": G,
                        "l2": "flushed between steps (256 MiB write, outside the timed events)",
                        "timing": "CUDA events per step on the launching stream around one CUDA graph of the "
-                                 "step (attention, split-job merge, sample head, gate), split by an event "
+                                 "step (attention, sample head, gate), split by an event "
                                  "recorded inside it" if one_graph else
                                  "CUDA events per step around the attention graph and the sample-head/gate graph",
                        "parallelism": f"replicas x{world}"},
             "step_hbm_gbs": step_gbs, "step_hbm_frac": step_gbs / peak,
             "step_algorithmic_bytes": step_bytes,
             "kernels_ms": {"attention": mean_attn, "sample_head_and_gate": sum(hg_ms) / len(hg_ms)},
-            "roofline": {"bound": "hbm", "kernel": "attn_tc_kernel<128> + attn_merge_kernel<128>", "achieved": attn_gbs,
+            "roofline": {"bound": "hbm", "kernel": "attn_tc_kernel<128, 4>", "achieved": attn_gbs,
                          "peak": peak, "unit": "GB/s", "frac": attn_gbs / peak, "traffic": traffic,
                          "algorithmic_bytes": attn_bytes, "peak_source": peak_kind},
             "cpu_baseline": cpu,

@@ -87,7 +87,7 @@ typedef struct {
   int32_t num_pages;         /* pages in each of the K and V pools              */
   int32_t max_prompt_pages;  /* columns of prompt_block_table (>= 1)            */
   int32_t max_suffix_pages;  /* columns of suffix_block_table (>= 1)            */
-  int32_t num_ctas;          /* persistent blocks; 0 = one per SM of the device  */
+  int32_t num_ctas;          /* persistent blocks (<= 65535); 0 = one per SM     */
   int32_t reserved;          /* must be 0                                       */
 } rgd_attn_shape;
 
@@ -117,11 +117,18 @@ size_t rgd_prefix_decode_attn_workspace_size(const rgd_attn_shape* shape);
  *   softmax_scale      > 0 (1/sqrt(D) for standard attention)
  *   out                bf16 [R, Hq, D]; lse float [R, Hq] or NULL
  *   workspace          device memory of rgd_prefix_decode_attn_workspace_size()
- *                      bytes, 256-byte aligned, contents arbitrary (a call
- *                      reads only what it wrote there).  Calls that share a
- *                      workspace must not overlap in time.
- * Two kernels run on `stream`: the attention kernel and a small merge of the
- * jobs that were split across blocks.
+ *                      bytes, 256-byte aligned, zero-filled before its first
+ *                      use.  It starts with one int32 counter per (group, kv
+ *                      head) job, which every call leaves at zero again unless
+ *                      it reports RGD_DEV_WAIT_TIMEOUT (then zero-fill it before
+ *                      reuse); the rest is scratch that a call writes before
+ *                      reading.  Calls that share a workspace must not overlap
+ *                      in time.
+ * One kernel runs on `stream`.  A job split across blocks is merged by the
+ * block holding its first page, which waits (bounded) for the job's other
+ * pieces; those are the first pieces of later blocks and wait on no other
+ * block, so the wait ends as long as blocks start in index order (num_ctas
+ * above the number of blocks the device holds at once relies on that).
  * A group with prompt_len 0 and a row with suffix_len 0 are valid; a row with
  * neither gets out = 0, lse = -inf.  Page ids outside [0, num_pages) read as
  * zeros and set RGD_DEV_BAD_PAGE.  Lengths beyond the table are rejected on the
@@ -148,9 +155,12 @@ int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf16* q,
  *   - The first call on a device looks up the array's device address (once per
  *     device, with that device current); make that first call before any stream
  *     capture.
- *   - Nothing is allocated or cleared: a call reads only scratch values that it
- *     wrote itself.  Every call shares the one array, so calls that overlap on
- *     the GPU (other streams, other threads) race: serialise them. */
+ *   - Nothing is allocated or cleared: the array starts zeroed when the library
+ *     is loaded and every call leaves its job counters at zero, unless it
+ *     reports RGD_DEV_WAIT_TIMEOUT (after which this entry point must not be
+ *     used again in the process).  Every call shares the one array, so calls
+ *     that overlap on the GPU (other streams, other threads) race: serialise
+ *     them. */
 int rgd_prefix_decode_attn_noalloc(const rgd_attn_shape* shape, const rgd_bf16* q,
                                    const rgd_bf16* k_pages, const rgd_bf16* v_pages,
                                    const int32_t* prompt_block_table, const int32_t* prompt_len,

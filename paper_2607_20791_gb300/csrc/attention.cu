@@ -14,8 +14,11 @@
 // the grid's persistent blocks (one per SM) each take an equal contiguous range
 // of pages.  A job split across blocks leaves a partial (o, m, l) in workspace
 // slot (block + job) -- distinct for every piece, since block ranges are ordered
-// like the jobs -- and a second, small kernel merges each split job's partials
-// by log-sum-exp (Sec. 3's shared-prefix split is the same identity).
+// like the jobs -- and takes a ticket; the block holding the job's last piece
+// to finish merges the partials by log-sum-exp (Sec. 3's shared-prefix split is
+// the same identity).  Only the two jobs at the ends of a block's range can be
+// split, and a block works on those two first, so the merges happen early and
+// overlap the rest of the block's work.
 //
 // Inside a block (608 threads) the tensor memory holds Q, S / P and O, so the
 // tensor cores read only K and V from shared memory -- the bytes that come from
@@ -109,8 +112,9 @@ struct AttnParams {
   __nv_bfloat16* out;
   float* lse;
   float* slot_o;    // [(C + J - 1) * nq, D]
-  float2* slot_ml;  // [(C + J - 1) * nq]
-  int32_t* gpre_ws; // [G + 1] page-count prefix, written by block 0 for the merge
+  float2* slot_ml;  // [(C + J - 1) * ml_stride(nq)]
+  int32_t* ticket;  // [J] pieces of a split job that have finished (zero between calls)
+  int npref;        // partner pieces whose partials fit the prefetch area (0..2)
   int32_t* dev_status;
   int32_t G, rpg, Hq, Hkv, gq, num_pages, max_pp, max_sp;
   int32_t nq, nslots, C;
@@ -120,8 +124,18 @@ struct AttnParams {
 // Shared-memory carve-up (identical on host and device).  The ring is 1024-byte
 // aligned: the 128-byte swizzle repeats every 8 rows of 128 bytes.
 struct SmemLayout {
-  int ring, red, gpre, gact, desc, rowbits, total;
+  int ring, red, gpre, gact, desc, rowbits, pref, total;
 };
+
+// Partial (m, l) pairs are stored nq rounded up to even per piece, so that
+// every piece's pairs start on a 16-byte boundary (bulk copies).
+__host__ __device__ constexpr int ml_stride(int nq) { return (nq + 1) & ~1; }
+
+// Shared memory for one partner piece's partial result, prefetched by the block
+// that will merge a split job: O rows padded to D + 4 floats (conflict-free
+// row-per-lane reads), then the (m, l) pairs.
+template <int D>
+__host__ __device__ constexpr int pref_bytes(int nq) { return nq * (D + 4) * 4 + ml_stride(nq) * 8; }
 
 __host__ __device__ inline int align_up(int x, int a) { return (x + a - 1) / a * a; }
 
@@ -135,17 +149,18 @@ __host__ __device__ constexpr int slot_bytes() {
 }
 
 template <int D>
-__host__ __device__ inline SmemLayout smem_layout(int nslots, int G, int R) {
+__host__ __device__ inline SmemLayout smem_layout(int nslots, int G, int R, int nq, int npref) {
   SmemLayout L;
   L.ring = 0;
   L.red = nslots * slot_bytes<D>();
   // row-max exchange (2 buffers), row sums and running maxima of 2 pieces, O
-  // staging for the copies >= 1 (at most 3 warps x 16 columns x 32 lanes)
-  L.gpre = L.red + (2 * 4 * kRows + 2 * 4 * kRows + 2 * kRows + 3 * 4 * 32 * 4) * 4;
+  // staging for the copies >= 1 (2 buffers of at most 3 warps x 16 columns x 32 lanes)
+  L.gpre = L.red + (2 * 4 * kRows + 2 * 4 * kRows + 2 * kRows + 2 * 3 * 4 * 32 * 4) * 4;
   L.gact = align_up(L.gpre + (G + 1) * 4, 16);
   L.desc = align_up(L.gact + G * 4, 16);
   L.rowbits = align_up(L.desc + nslots * kGroupPages * 4, 16);  // one bit per row: active
-  L.total = align_up(L.rowbits + (R + 31) / 32 * 4, 16) + 1024;  // + slack for the 1024-byte aligned base
+  L.pref = align_up(L.rowbits + (R + 31) / 32 * 4, 16);
+  L.total = L.pref + npref * pref_bytes<D>(nq) + 1024;  // + slack for the 1024-byte aligned base
   return L;
 }
 
@@ -197,6 +212,53 @@ __device__ Job next_job(const AttnParams& p, const int32_t* gpre, Job j) {
 // Block whose page range contains global page x (ranges [floor(cT/C), floor((c+1)T/C))).
 __device__ __forceinline__ int cta_of(int64_t x, int64_t T, int C) { return (int)(((x + 1) * C - 1) / T); }
 
+// A block's job pieces in the order it works on them: the job at the start of
+// its range, then the job at the end, then the whole jobs in between.  Only the
+// two end jobs can be split with a neighbouring block, so every split job is
+// finished early in both of its blocks and is merged off their critical paths.
+struct PieceIter {
+  Job j0, jl;       // first and last job of the range
+  int n0, nl;       // their pages in the range (nl = 0: the range holds one job)
+  int64_t mid_end;  // global page where the middle jobs end
+};
+
+__device__ PieceIter piece_iter(const AttnParams& p, const int32_t* gpre, int64_t b, int64_t e) {
+  PieceIter it;
+  it.j0 = job_at(p, gpre, b);
+  it.n0 = (int)(min(e, it.j0.start + it.j0.n) - b);
+  it.jl = it.j0;
+  it.nl = 0;
+  it.mid_end = e;
+  if (b + it.n0 < e) {
+    it.jl = job_at(p, gpre, e - 1);
+    it.nl = (int)(e - it.jl.start);
+    it.mid_end = it.jl.start;
+  }
+  return it;
+}
+
+// Piece k (>= 1) after piece k - 1 = (cur, n); false when there is none.
+__device__ bool next_piece(const AttnParams& p, const int32_t* gpre, const PieceIter& it, int k, Job& cur, int& n) {
+  if (k == 1) {
+    if (it.nl == 0) return false;
+    cur = it.jl;
+    n = it.nl;
+    return true;
+  }
+  const Job nx = next_job(p, gpre, k == 2 ? it.j0 : cur);
+  if (nx.start >= it.mid_end) return false;
+  cur = nx;
+  n = nx.n;
+  return true;
+}
+
+// Global page of position i of a block's page sequence (pieces in PieceIter order).
+__device__ __forceinline__ int64_t seq_page(const PieceIter& it, int64_t b, int64_t i) {
+  if (i < it.n0) return b + i;
+  if (i < it.n0 + it.nl) return it.jl.start + (i - it.n0);
+  return b + it.n0 + (i - it.n0 - it.nl);
+}
+
 // Bounded wait that also gives up as soon as another role has given up.
 // A waiting thread sleeps inside try_wait (woken when the phase completes), so
 // warps parked on a barrier take no issue slots from the working ones.
@@ -234,6 +296,68 @@ __device__ __forceinline__ bool wait_slot_gen(int32_t* gen, int32_t want, volati
   }
 }
 
+// Merge of split job jj's partials (pieces first..last, workspace slots
+// piece + jj) by n_threads threads, thread et taking items et, et + n_threads,
+// ... (item = 4 output columns of one query): with piece s holding the
+// unnormalised o_s and (m_s, l_s) in log2 units,
+//   out = sum_s 2^(m_s - M) o_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s.
+// kP pieces' loads are issued together (more registers, fewer round trips).
+template <int D, int kP>
+__device__ __forceinline__ void merge_job(const AttnParams& p, const uint32_t* rowbits, Job jb, int jj, int first,
+                                       int last, int et, int n_threads) {
+  constexpr int kC4 = D / 4;
+  const int nq = p.nq, gq = p.gq;
+  for (int item = et; item < nq * kC4; item += n_threads) {
+    const int i = item / kC4, c4 = item % kC4;
+    const int rr2 = jb.g * p.rpg + i / gq, hq2 = jb.h * gq + i % gq;
+    if (!((rowbits[rr2 >> 5] >> (rr2 & 31)) & 1u)) continue;
+    float Mm = -INFINITY, Lm = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int c0 = first; c0 <= last; c0 += kP) {
+      float2 ml[kP];
+      float4 v[kP];
+#pragma unroll
+      for (int t = 0; t < kP; ++t) {
+        if (c0 + t <= last) {
+          const int64_t sl = (int64_t)(c0 + t) + jj;
+          ml[t] = __ldcg(p.slot_ml + sl * ml_stride(nq) + i);
+          v[t] = __ldcg(reinterpret_cast<const float4*>(p.slot_o + (sl * nq + i) * D) + c4);
+        } else {
+          ml[t] = make_float2(-INFINITY, 0.f);
+        }
+      }
+      float Mn = Mm;
+#pragma unroll
+      for (int t = 0; t < kP; ++t)
+        if (ml[t].y != 0.f) Mn = fmaxf(Mn, ml[t].x);
+      if (Mn == -INFINITY) continue;
+      const float f = (Mm == -INFINITY) ? 0.f : exp2f(Mm - Mn);
+      Lm *= f;
+      acc.x *= f;
+      acc.y *= f;
+      acc.z *= f;
+      acc.w *= f;
+#pragma unroll
+      for (int t = 0; t < kP; ++t) {
+        if (ml[t].y == 0.f) continue;
+        const float wt = exp2f(ml[t].x - Mn);
+        Lm += wt * ml[t].y;
+        acc.x += wt * v[t].x;
+        acc.y += wt * v[t].y;
+        acc.z += wt * v[t].z;
+        acc.w += wt * v[t].w;
+      }
+      Mm = Mn;
+    }
+    const float iv = Lm > 0.f ? 1.f / Lm : 0.f;
+    uint2 pk2;
+    pk2.x = pack_bf16x2(acc.x * iv, acc.y * iv);
+    pk2.y = pack_bf16x2(acc.z * iv, acc.w * iv);
+    reinterpret_cast<uint2*>(p.out + ((int64_t)rr2 * p.Hq + hq2) * D)[c4] = pk2;
+    if (p.lse && c4 == 0) p.lse[(int64_t)rr2 * p.Hq + hq2] = Lm > 0.f ? (Mm + log2f(Lm)) * kLn2 : -INFINITY;
+  }
+}
+
 template <int D, int R>
 __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
@@ -246,18 +370,19 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
   constexpr uint32_t kIdescPV = idesc_bf16_f32(kRows, D, 0, 1);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const SmemLayout L = smem_layout<D>(p.nslots, p.G, p.G * p.rpg);
+  const SmemLayout L = smem_layout<D>(p.nslots, p.G, p.G * p.rpg, p.nq, p.npref);
   uint32_t* rowbits = reinterpret_cast<uint32_t*>(smem + L.rowbits);
   int32_t* gpre = reinterpret_cast<int32_t*>(smem + L.gpre);
   uint32_t* descs = reinterpret_cast<uint32_t*>(smem + L.desc);
   __shared__ uint64_t full_bar[kMaxSlots], empty_bar[kMaxSlots];
   __shared__ uint64_t s_full[kSBufs], s_empty[kSBufs], p_full[kPBufs], p_empty[kPBufs];
   __shared__ uint64_t q_full, q_empty, o_full[2], o_free[2], ml_full[2], ml_empty[2], mma_done[2];
+  __shared__ uint64_t pref_bar;  // a split job's partner partials have landed in shared memory
   using Rl = Roles<R>;
   constexpr int kAttnThreads = Rl::kThreads;
   constexpr int kSoftThreads = Rl::kSoft * 32;
   constexpr int kProducerWarp = Rl::kProducer, kMmaWarp = Rl::kMma, kPvWarp = Rl::kPv;
-  __shared__ int32_t s_abort, s_issued, s_wsum[kMaxAttnWarps];
+  __shared__ int32_t s_abort, s_issued, s_last, s_pref_n, s_wsum[kMaxAttnWarps];
   __shared__ int32_t s_slot_gen[kMaxSlots];  // the last group that entered each ring slot
   __shared__ uint32_t s_tmem;
   volatile int32_t* abort_flag = &s_abort;
@@ -298,8 +423,10 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
     }
     mbar_init(&mma_done[0], 1);
     mbar_init(&mma_done[1], 1);
+    mbar_init(&pref_bar, 1);
     s_abort = 0;
     s_issued = 0;
+    s_pref_n = 0;  // partner prefetches issued
     for (int i = 0; i < kMaxSlots; ++i) s_slot_gen[i] = -1;
     fence_mbar_init();
   }
@@ -365,16 +492,16 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
     }
   }
   __syncthreads();
-  if (c == 0)
-    for (int g = tid; g <= p.G; g += kAttnThreads) p.gpre_ws[g] = gpre[g];
-  // the merge kernel may be launched now; it waits for this grid to complete
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int64_t T = (int64_t)p.Hkv * gpre[p.G];
   // pages are divided over Ceff = min(C, T) blocks so that every working block
   // has at least one page (a job's pieces are then exactly the blocks first..last)
   const int Ceff = (int)min((int64_t)p.C, T);
   const int64_t b = c < Ceff ? (int64_t)c * T / Ceff : T;
   const int64_t e = c < Ceff ? (int64_t)(c + 1) * T / Ceff : T;
+  // the piece order, kept in shared memory (read at piece boundaries only)
+  __shared__ PieceIter s_it;
+  if (tid == 0 && b < e) s_it = piece_iter(p, gpre, b, e);
+  __syncthreads();
 
   if (warp >= kProducerWarp && warp < kProducerWarp + kProducerWarps) {
     // ============================ producers ===========================
@@ -398,11 +525,12 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
         prefetch_tensormap(&tmV);
       }
       const uint64_t pol = policy_evict_first();
-      int gbase = 0;  // groups started before xb
+      const PieceIter& it = s_it;
+      int gbase = 0;  // groups started before sequence position ib
       int rnd = 0;
-      for (int64_t xb = b; xb < e; xb += 32, ++rnd) {
-        const int64_t x = xb + lane;
-        const bool valid = x < e;
+      for (int64_t ib = 0; ib < e - b; ib += 32, ++rnd) {
+        const bool valid = ib + lane < e - b;
+        const int64_t x = valid ? seq_page(it, b, ib + lane) : b;
         const bool mine = (rnd % kProducerWarps) == pw;
         int32_t page = -1, tok = 0, rowsel = -1, hh = 0, jpos = 0, ng = 0;
         if (valid) {
@@ -498,10 +626,10 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
       const uint64_t k_d = smem_desc(sbase, 1024, 1024, 2);
       int gi = 0, pc = 0;
       bool ok = true;
-      Job cur = job_at(p, gpre, b);
-      int64_t x0 = b;
-      while (ok && x0 < e) {
-        const int n_in = (int)(min(e, cur.start + cur.n) - x0);
+      const PieceIter& it = s_it;
+      Job cur = it.j0;
+      int n_in = it.n0;
+      for (bool more = b < e; ok && more; more = next_piece(p, gpre, it, pc, cur, n_in)) {
         if (!wait_or_abort(&q_full, (uint32_t)pc & 1u, abort_flag)) break;
         tc_fence_after();
         const uint32_t qa = tmem + kQCol;
@@ -532,8 +660,6 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
           ++gi;
         }
         ++pc;
-        x0 += n_in;
-        if (x0 < e) cur = next_job(p, gpre, cur);
       }
     }
   } else if (warp == kPvWarp) {
@@ -545,10 +671,10 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
       const uint64_t v_d = smem_desc(sbase, D == 128 ? kVLbo : 1024, D == 128 ? kVSbo : 1024, 2);
       int gi = 0, pc = 0;
       bool ok = true;
-      Job cur = job_at(p, gpre, b);
-      int64_t x0 = b;
-      while (ok && x0 < e) {
-        const int n_in = (int)(min(e, cur.start + cur.n) - x0);
+      const PieceIter& it = s_it;
+      Job cur = it.j0;
+      int n_in = it.n0;
+      for (bool more = b < e; ok && more; more = next_piece(p, gpre, it, pc, cur, n_in)) {
         for (int k0 = 0; k0 < n_in; k0 += kGroupPages) {
           const int ng = min(kGroupPages, n_in - k0);
           const int pb = gi % kPBufs;
@@ -579,8 +705,6 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
           ++gi;
         }
         ++pc;
-        x0 += n_in;
-        if (x0 < e) cur = next_job(p, gpre, cur);
       }
     }
   } else {
@@ -616,8 +740,11 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
     float* rmax = reinterpret_cast<float*>(smem + L.red);  // [2][4][128] page-slot maxima
     float* rsum = rmax + 2 * 4 * kRows;                    // [2 pieces][4][128] page-slot row sums
     float* mfin = rsum + 2 * 4 * kRows;                    // [2 pieces][128] running max at the piece end
-    float4* stage = reinterpret_cast<float4*>(mfin + 2 * kRows);  // [<= 9][4][32] O columns of copies >= 1
+    float4* stage = reinterpret_cast<float4*>(mfin + 2 * kRows);  // [2][<= 3][4][32] O columns of copies >= 1
     const int ocols = D / W;                   // O columns rescaled by each softmax warp of a quarter
+    float* pref_o = reinterpret_cast<float*>(smem + L.pref);                        // [npref][nq][D + 4]
+    float2* pref_ml = reinterpret_cast<float2*>(pref_o + p.npref * nq * (D + 4));   // [npref][ml_stride(nq)]
+    int n_pref = 0;  // prefetches completed (the parity of pref_bar)
     constexpr int kChunks = D / 16;            // 16-column chunks of O (and 8-column chunks of Q)
     // warp-uniform bounded wait (TMEM loads and stores that follow are warp-collective)
     auto wwait = [&](uint64_t* bar, uint32_t parity, volatile int32_t* flag) {
@@ -626,7 +753,8 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
     // Q of job jb: this epilogue warp's share of its rows' query columns (8-column
     // chunks ei, ei + NE, ...), loaded first; then, if `after` is set, the wait for
     // the last QK of the piece before, which frees the single Q buffer
-    auto write_q = [&](const Job& jb, bool after, uint32_t parity) {
+    // (the loads are issued before the wait for q_empty, which `waitf` does)
+    auto write_q = [&](const Job& jb, bool after, uint32_t parity, auto&& waitf) {
       constexpr int kMaxChunks = (kChunks + NE - 1) / NE;
       uint4 qv[2 * kMaxChunks];
       int n = 0;
@@ -646,7 +774,7 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
         }
       }
       bool fine = true;
-      if (after && !wwait(&q_empty, parity, abort_flag)) fine = false;
+      if (after && !waitf(&q_empty, parity)) fine = false;
       if (fine) {
         tc_fence_after();
 #pragma unroll
@@ -803,115 +931,348 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(&ml_full[ob]);
           };
+    // Merge of a split job's partials by the epilogue threads, one piece at a
+    // time: bulk copies bring the piece's partial into the prefetch area and
+    // each thread folds it into its items (item = 4 output columns of one
+    // query), kU items at a time: with piece s holding the unnormalised o_s and
+    // (m_s, l_s) in log2 units, out = sum 2^(m_s - M) o_s / sum 2^(m_s - M) l_s.
+    auto merge_staged = [&](const Job& jb, int jj, int first, int last, int et, int n_et, bool copier) {
+      constexpr int kU = R == 4 ? 8 : 2;  // (more fit in the registers of the 4-copy layout only)
+      const int mls = ml_stride(nq), n4 = nq * (D / 4);
+      bool good = true;  // no wait has given up (the barriers below are passed regardless)
+      for (int b0 = 0; b0 < n4; b0 += kU * n_et) {  // (the same trip counts in every thread)
+        const int base = b0 + et;
+        float Mm[kU], Lm[kU];
+        float4 acc[kU];
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+          Mm[u] = -INFINITY;
+          Lm[u] = 0.f;
+          acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        for (int s2 = first; s2 <= last; ++s2) {
+          const int64_t sl = (int64_t)s2 + jj;
+          if (copier && __all_sync(0xffffffffu, good && !*abort_flag)) {
+            if (lane == 0) {
+              mbar_arrive_expect_tx(&pref_bar, (uint32_t)(nq * D * 4 + mls * 8));
+              ++s_pref_n;
+            }
+            __syncwarp();
+            fence_proxy_async_global();
+            for (int i = lane; i <= nq; i += 32) {
+              if (i < nq) bulk_load(pref_o + i * (D + 4), p.slot_o + (sl * nq + i) * D, D * 4, &pref_bar);
+              else bulk_load(pref_ml, p.slot_ml + sl * mls, mls * 8, &pref_bar);
+            }
+          }
+          good = wwait(&pref_bar, (uint32_t)n_pref & 1u, abort_flag) && good;  // (after an abort: at once)
+          ++n_pref;
+#pragma unroll
+          for (int u = 0; u < kU; ++u) {
+            const int it = base + u * n_et;
+            if (!good || it >= n4) break;
+            const int i = it / (D / 4), c4 = it % (D / 4);
+            const float2 ml = pref_ml[i];
+            if (ml.y == 0.f) continue;
+            const float4 v = reinterpret_cast<const float4*>(pref_o + i * (D + 4))[c4];
+            const float Mn = fmaxf(Mm[u], ml.x);
+            const float f = Mm[u] == -INFINITY ? 0.f : exp2f(Mm[u] - Mn), w = exp2f(ml.x - Mn);
+            Lm[u] = Lm[u] * f + w * ml.y;
+            acc[u].x = acc[u].x * f + w * v.x;
+            acc[u].y = acc[u].y * f + w * v.y;
+            acc[u].z = acc[u].z * f + w * v.z;
+            acc[u].w = acc[u].w * f + w * v.w;
+            Mm[u] = Mn;
+          }
+          epi_sync();  // the area is read before the next piece's copies
+        }
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+          const int it = base + u * n_et;
+          if (!good || it >= n4) break;  // (after an abort the outputs are not written)
+          const int i = it / (D / 4), c4 = it % (D / 4);
+          const int rr2 = jb.g * p.rpg + i / gq, hq2 = jb.h * gq + i % gq;
+          if (!((rowbits[rr2 >> 5] >> (rr2 & 31)) & 1u)) continue;
+          const float iv = Lm[u] > 0.f ? 1.f / Lm[u] : 0.f;
+          uint2 pk2;
+          pk2.x = pack_bf16x2(acc[u].x * iv, acc[u].y * iv);
+          pk2.y = pack_bf16x2(acc[u].z * iv, acc[u].w * iv);
+          reinterpret_cast<uint2*>(p.out + ((int64_t)rr2 * p.Hq + hq2) * D)[c4] = pk2;
+          if (p.lse && c4 == 0)
+            p.lse[(int64_t)rr2 * p.Hq + hq2] = Lm[u] > 0.f ? (Mm[u] + log2f(Lm[u])) * kLn2 : -INFINITY;
+        }
+      }
+    };
     // the next piece's Q, then this piece's end (epilogue warps)
     auto run_epilogue = [&](const Job& cur, int pc, bool more, const Job& nxt) {
       const int j = cur.g * p.Hkv + cur.h;
       const int ob = pc & 1;
       const uint32_t ocol = kOCol + ob * kOStride;
-        // ---- the next piece's Q, once this piece's last QK is done ----
-        if (more && !write_q(nxt, true, (uint32_t)pc & 1u)) ok = false;
-        // ---- this piece's epilogue: O is final once its last PV completes ----
-        const int first = cta_of(cur.start, T, Ceff), last = cta_of(cur.start + cur.n - 1, T, Ceff);
-        const int rr = r < nq ? cur.g * p.rpg + r / gq : 0, hq = r < nq ? cur.h * gq + r % gq : 0;
-        const bool mine_row = r < nq && cp == 0;
-        const bool write_row = mine_row && ((rowbits[rr >> 5] >> (rr & 31)) & 1u);
-        if (ok && !wwait(&o_full[ob], (uint32_t)(pc >> 1) & 1u, abort_flag)) ok = false;
-        if (ok && !wwait(&ml_full[ob], (uint32_t)(pc >> 1) & 1u, abort_flag)) ok = false;
-        tc_fence_after();
-        // the copies' running maxima and row sums -> the piece's max M and sum L;
-        // copy c's O is weighted by 2^(m_c - M)
-        float M = -INFINITY, Ls = 0.f;
-        for (int c2 = 0; c2 < R; ++c2) M = fmaxf(M, mfin[ob * kRows + (c2 * qpc + rb) * 32 + lane]);
-        for (int c2 = 0; c2 < R; ++c2) {
-          const int ln = (c2 * qpc + rb) * 32 + lane;
-          float Lc = 0.f;
-          for (int w = 0; w < W; ++w) Lc += rsum[(ob * 4 + w) * kRows + ln];
-          const float mc = mfin[ob * kRows + ln];
-          if (mc != -INFINITY) Ls += exp2f(mc - M) * Lc;
+      const int first = cta_of(cur.start, T, Ceff), last = cta_of(cur.start + cur.n - 1, T, Ceff);
+      const int rr = r < nq ? cur.g * p.rpg + r / gq : 0, hq = r < nq ? cur.h * gq + r % gq : 0;
+      const bool mine_row = r < nq && cp == 0;
+      const bool write_row = mine_row && ((rowbits[rr >> 5] >> (rr & 31)) & 1u);
+      const int et = (ei * (R * qpc) + qd) * 32 + lane;  // index among the epilogue threads
+      const int n_et = n_epi * 32;
+      const bool watcher = ei == 0 && qd == 0;           // the warp holding et == 0
+      // A split job is merged by the block holding its first page (the merger);
+      // its other pieces (each the first piece of its own block, so never
+      // behind a wait on another block) write a partial and count themselves
+      // in the job's ticket (an aborted piece also in the high half).  The
+      // merger's watcher warp watches the ticket while this piece runs and,
+      // once the count is complete, has bulk copies bring the partials into
+      // shared memory; the merger then folds them into its own O on the way out.
+      const bool split = first != last;
+      const int nparts = last - first;  // the job's other pieces
+      const bool merger = split && c == first;
+      const bool staged = merger && nparts <= p.npref;  // the partials fit the prefetch area
+      auto issue_prefetch = [&]() {                       // (the watcher warp, all lanes)
+        const int mls = ml_stride(nq);
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&pref_bar, (uint32_t)(nparts * (nq * D * 4 + mls * 8)));
+          ++s_pref_n;
         }
-        const float mself = mfin[ob * kRows + tlane];
-        const float wself = mself == -INFINITY ? 0.f : exp2f(mself - M);
         __syncwarp();
-        if (lane == 0) mbar_arrive(&ml_empty[ob]);  // the (m, l) slot has been read
-        const int64_t s_idx = (int64_t)c + j;
-        const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-        // after an abort the piece's outputs are not written (the status word says so)
-        const bool out_ok = __all_sync(0xffffffffu, ok && !*abort_flag);
-        // O in 16-column chunks: epilogue warp ei of a quarter takes chunks ei,
-        // ei + NE, ...; copies >= 1 pass theirs to copy 0 through shared memory
-        constexpr int rounds = (kChunks + NE - 1) / NE;
-        const int my_stage = ((cp - 1) * qpc + rb) * NE + ei;  // (for copies >= 1)
-#pragma unroll 1
-        for (int rd = 0; rd < rounds; ++rd) {
-          const int ch = ei + rd * NE;
-          const bool has = ch < kChunks && out_ok;
-          const int col = ch * 16;
-          float o[16];
-          if (has) {
-            uint32_t raw[16];
-            tmem_ld16(tl + ocol + col, raw);
-            tmem_ld_wait();
-#pragma unroll
-            for (int t = 0; t < 16; ++t) o[t] = __uint_as_float(raw[t]) * wself;
-          }
-          if (R > 1) {
-            if (rd > 0) epi_sync();  // the previous round's staging has been read
-            if (cp > 0 && has) {
-#pragma unroll
-              for (int t = 0; t < 4; ++t)
-                stage[(my_stage * 4 + t) * 32 + lane] = make_float4(o[4 * t], o[4 * t + 1], o[4 * t + 2], o[4 * t + 3]);
+        fence_proxy_async_global();  // the partials were seen by the generic proxy (the acquire)
+        for (int it = lane; it < nparts * (nq + 1); it += 32) {
+          const int k = it / (nq + 1), i = it % (nq + 1);
+          const int64_t sl = (int64_t)(first + k + 1) + j;  // the k-th other piece's slot
+          if (i < nq) bulk_load(pref_o + (k * nq + i) * (D + 4), p.slot_o + (sl * nq + i) * D, D * 4, &pref_bar);
+          else bulk_load(pref_ml + k * mls, p.slot_ml + sl * mls, mls * 8, &pref_bar);
+        }
+      };
+      // (watcher) the ticket once its count is complete (0: not seen yet), and
+      // whether the partner copies are on their way
+      int tk = 0;
+      bool issued = false;
+      const bool polling = staged && watcher;
+      // the ticket read is consumed a few sleeps later, so that a wait never
+      // stalls on it once its barrier has completed
+      int pend = polling && lane == 0 ? ld_acquire_gpu(p.ticket + j) : 0;
+      auto seen = [&](int t) {
+        if ((t & 0xffff) != nparts) return false;
+        tk = t;
+        if (staged && (t >> 16) == 0 && __all_sync(0xffffffffu, ok)) {  // (only staged partials fit the area)
+          issue_prefetch();
+          issued = true;
+        }
+        return true;
+      };
+      // A bounded wait on `bar`, during which the watcher polls the ticket.
+      auto wait_polling = [&](uint64_t* bar, uint32_t par) -> bool {
+        if (!polling || !__all_sync(0xffffffffu, ok)) return ok && wwait(bar, par, abort_flag);
+        // (a non-blocking test and short sleeps: a blocking try_wait would
+        // return only once the phase completes)
+        const uint64_t t0 = globaltimer_ns();
+        for (uint32_t i = 1;; ++i) {
+          if (__any_sync(0xffffffffu, mbar_test_wait(bar, par))) return true;
+          if (tk == 0 && (i & 7u) == 0 && !seen(__shfl_sync(0xffffffffu, pend, 0)) && lane == 0)
+            pend = ld_acquire_gpu(p.ticket + j);
+          __nanosleep(200);
+          if ((i & 63u) == 0) {  // (warp-uniform exits: the loop holds warp collectives)
+            if (__any_sync(0xffffffffu, *abort_flag != 0)) return false;
+            if (__any_sync(0xffffffffu, globaltimer_ns() - t0 > kWaitLimitNs)) {
+              *abort_flag = 1;
+              return false;
             }
-            epi_sync();
-            if (cp == 0 && has) {
-#pragma unroll 1
-              for (int c2 = 1; c2 < R; ++c2) {
-                const float4* src4 = stage + ((((c2 - 1) * qpc + rb) * NE + ei) * 4) * 32 + lane;
+          }
+        }
+      };
+      // (watcher) Bounded wait until the job's other pieces have all counted
+      // themselves: they never wait on this block, so it ends; it is also
+      // waited for after an abort, so that the merger can clear the ticket.
+      auto wait_ticket = [&]() {
+        const uint64_t t0 = globaltimer_ns();
+        while (tk == 0) {
+          if (seen(__shfl_sync(0xffffffffu, lane == 0 ? ld_acquire_gpu(p.ticket + j) : 0, 0))) break;
+          if (__any_sync(0xffffffffu, globaltimer_ns() - t0 > kWaitLimitNs)) {
+            *abort_flag = 1;
+            tk = -1;
+            break;
+          }
+          __nanosleep(256);
+        }
+      };
+      // ---- the next piece's Q, once this piece's last QK is done ----
+      if (more && !write_q(nxt, true, (uint32_t)pc & 1u, wait_polling)) ok = false;
+      // ---- this piece's epilogue: O is final once its last PV completes ----
+      if (!wait_polling(&o_full[ob], (uint32_t)(pc >> 1) & 1u)) ok = false;
+      if (ok && !wwait(&ml_full[ob], (uint32_t)(pc >> 1) & 1u, abort_flag)) ok = false;
+      tc_fence_after();
+      // the copies' running maxima and row sums -> the piece's max M and sum L;
+      // copy c's O is weighted by 2^(m_c - M)
+      float M = -INFINITY, Ls = 0.f;
+      for (int c2 = 0; c2 < R; ++c2) M = fmaxf(M, mfin[ob * kRows + (c2 * qpc + rb) * 32 + lane]);
+      for (int c2 = 0; c2 < R; ++c2) {
+        const int ln = (c2 * qpc + rb) * 32 + lane;
+        float Lc = 0.f;
+        for (int w = 0; w < W; ++w) Lc += rsum[(ob * 4 + w) * kRows + ln];
+        const float mc = mfin[ob * kRows + ln];
+        if (mc != -INFINITY) Ls += exp2f(mc - M) * Lc;
+      }
+      const float mself = mfin[ob * kRows + tlane];
+      const float wself = mself == -INFINITY ? 0.f : exp2f(mself - M);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ml_empty[ob]);  // the (m, l) slot has been read
+      const int64_t s_idx = (int64_t)c + j;
+      // fused: a merger whose partners' partials are (being) staged folds them
+      // in here, with its own O still in registers
+      bool fused = false, partners_ok = true;
+      if (staged) {
+        if (watcher) {
+          wait_ticket();
+          if (lane == 0) s_last = issued ? 1 : 0;  // 0: a piece (or this block) gave up
+        }
+        epi_sync();
+        fused = true;
+        partners_ok = s_last == 1;
+        if (partners_ok) {
+          if (!wwait(&pref_bar, (uint32_t)n_pref & 1u, abort_flag)) ok = false;  // the partials have landed
+          ++n_pref;
+        }
+      }
+      // after an abort the piece's outputs are not written (the status word says so)
+      const bool out_ok = __all_sync(0xffffffffu, ok && !*abort_flag) && partners_ok;
+      // this piece's weight a and the partners' b_k in the merged softmax:
+      // out = (a o + sum_k b_k o_k) / (a L + sum_k b_k l_k)
+      float Mt = M, Lt = Ls, a = 1.f, bk[2] = {0.f, 0.f};
+      if (fused && out_ok && r < nq) {
+        Mt = Ls > 0.f ? M : -INFINITY;
+        float2 ml[2];
 #pragma unroll
-                for (int t = 0; t < 4; ++t) {
-                  const float4 v = src4[t * 32];
-                  o[4 * t] += v.x;
-                  o[4 * t + 1] += v.y;
-                  o[4 * t + 2] += v.z;
-                  o[4 * t + 3] += v.w;
-                }
+        for (int k = 0; k < 2; ++k) {
+          ml[k] = k < nparts ? pref_ml[k * ml_stride(nq) + r] : make_float2(-INFINITY, 0.f);
+          if (ml[k].y > 0.f) Mt = fmaxf(Mt, ml[k].x);
+        }
+        a = Ls > 0.f ? exp2f(M - Mt) : 0.f;
+        Lt = a * Ls;
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+          bk[k] = ml[k].y > 0.f ? exp2f(ml[k].x - Mt) : 0.f;
+          Lt += bk[k] * ml[k].y;
+        }
+      }
+      const float inv = Lt > 0.f ? 1.f / Lt : 0.f;
+      // O in 16-column chunks: epilogue warp ei of a quarter takes chunks ei,
+      // ei + NE, ...; copies >= 1 pass theirs to copy 0 through shared memory
+      constexpr int rounds = (kChunks + NE - 1) / NE;
+      const int my_stage = ((cp - 1) * qpc + rb) * NE + ei;  // (for copies >= 1)
+#pragma unroll 1
+      for (int rd = 0; rd < rounds; ++rd) {
+        const int ch = ei + rd * NE;
+        const bool has = ch < kChunks && out_ok;
+        const int col = ch * 16;
+        float o[16];
+        if (has) {
+          uint32_t raw[16];
+          tmem_ld16(tl + ocol + col, raw);
+          tmem_ld_wait();
+#pragma unroll
+          for (int t = 0; t < 16; ++t) o[t] = __uint_as_float(raw[t]) * wself;
+        }
+        if (R > 1) {
+          // double-buffered: a round's staging is rewritten two rounds later,
+          // after the next round's barrier, which copy 0 passes only once it
+          // has read it
+          float4* stg = stage + (rd & 1) * (3 * 4 * 32);
+          if (cp > 0 && has) {
+#pragma unroll
+            for (int t = 0; t < 4; ++t)
+              stg[(my_stage * 4 + t) * 32 + lane] = make_float4(o[4 * t], o[4 * t + 1], o[4 * t + 2], o[4 * t + 3]);
+          }
+          epi_sync();
+          if (cp == 0 && has) {
+#pragma unroll
+            for (int c2 = 1; c2 < R; ++c2) {
+              const float4* src4 = stg + ((((c2 - 1) * qpc + rb) * NE + ei) * 4) * 32 + lane;
+#pragma unroll
+              for (int t = 0; t < 4; ++t) {
+                const float4 v = src4[t * 32];
+                o[4 * t] += v.x;
+                o[4 * t + 1] += v.y;
+                o[4 * t + 2] += v.z;
+                o[4 * t + 3] += v.w;
               }
             }
           }
-          if (!has) continue;
-          if (first == last) {
-            if (write_row) {
-              uint4* dst = reinterpret_cast<uint4*>(p.out + ((int64_t)rr * p.Hq + hq) * D + col);
-              dst[0] = make_uint4(pack_bf16x2(o[0] * inv, o[1] * inv), pack_bf16x2(o[2] * inv, o[3] * inv),
-                                  pack_bf16x2(o[4] * inv, o[5] * inv), pack_bf16x2(o[6] * inv, o[7] * inv));
-              dst[1] = make_uint4(pack_bf16x2(o[8] * inv, o[9] * inv), pack_bf16x2(o[10] * inv, o[11] * inv),
-                                  pack_bf16x2(o[12] * inv, o[13] * inv), pack_bf16x2(o[14] * inv, o[15] * inv));
-            }
-          } else if (mine_row) {
-            float4* dst = reinterpret_cast<float4*>(p.slot_o + (s_idx * nq + r) * D + col);
+        }
+        if (!has) continue;
+        if (!split || fused) {
+          if (write_row) {
+            if (fused) {
 #pragma unroll
-            for (int t = 0; t < 4; ++t) dst[t] = make_float4(o[4 * t], o[4 * t + 1], o[4 * t + 2], o[4 * t + 3]);
+              for (int t = 0; t < 16; ++t) o[t] *= a;
+#pragma unroll
+              for (int k = 0; k < 2; ++k) {
+                if (k >= nparts) break;
+                const float4* src4 = reinterpret_cast<const float4*>(pref_o + (k * nq + r) * (D + 4) + col);
+#pragma unroll
+                for (int t = 0; t < 4; ++t) {
+                  const float4 v = src4[t];
+                  o[4 * t] += bk[k] * v.x;
+                  o[4 * t + 1] += bk[k] * v.y;
+                  o[4 * t + 2] += bk[k] * v.z;
+                  o[4 * t + 3] += bk[k] * v.w;
+                }
+              }
+            }
+            uint4* dst = reinterpret_cast<uint4*>(p.out + ((int64_t)rr * p.Hq + hq) * D + col);
+            dst[0] = make_uint4(pack_bf16x2(o[0] * inv, o[1] * inv), pack_bf16x2(o[2] * inv, o[3] * inv),
+                                pack_bf16x2(o[4] * inv, o[5] * inv), pack_bf16x2(o[6] * inv, o[7] * inv));
+            dst[1] = make_uint4(pack_bf16x2(o[8] * inv, o[9] * inv), pack_bf16x2(o[10] * inv, o[11] * inv),
+                                pack_bf16x2(o[12] * inv, o[13] * inv), pack_bf16x2(o[14] * inv, o[15] * inv));
           }
+        } else if (mine_row) {
+          float4* dst = reinterpret_cast<float4*>(p.slot_o + (s_idx * nq + r) * D + col);
+#pragma unroll
+          for (int t = 0; t < 4; ++t) dst[t] = make_float4(o[4 * t], o[4 * t + 1], o[4 * t + 2], o[4 * t + 3]);
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&o_free[ob]);  // this O buffer may take the piece after next
-        if (first == last) {
-          if (out_ok && ei == 0 && write_row && p.lse)
-            p.lse[(int64_t)rr * p.Hq + hq] = Ls > 0.f ? (M + log2f(Ls)) * kLn2 : -INFINITY;
-        } else if (out_ok && ei == 0 && mine_row) {
-          p.slot_ml[s_idx * nq + r] = make_float2(M, Ls);  // the merge kernel finishes the job
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&o_free[ob]);  // this O buffer may take the piece after next
+      if (!split || fused) {
+        if (out_ok && ei == 0 && write_row && p.lse)
+          p.lse[(int64_t)rr * p.Hq + hq] = Lt > 0.f ? (Mt + log2f(Lt)) * kLn2 : -INFINITY;
+        if (fused && et == 0) p.ticket[j] = 0;  // every other piece has counted itself
+        if (R > 1 || fused) epi_sync();         // staging and prefetch areas are reused at the next piece
+        return;
+      }
+      // this piece's partial, visible before its count
+      if (out_ok && ei == 0 && mine_row) p.slot_ml[s_idx * ml_stride(nq) + r] = make_float2(M, Ls);
+      __threadfence();
+      epi_sync();
+      if (!merger) {
+        if (et == 0) atomicAdd(p.ticket + j, out_ok && !*abort_flag ? 1 : 0x10001);
+        return;
+      }
+      // a merger whose partners' partials do not fit the prefetch area: once
+      // they have all counted themselves, merge every piece's partial
+      if (watcher) {
+        wait_ticket();
+        if (lane == 0) s_last = tk > 0 && (tk >> 16) == 0 && !*abort_flag ? 1 : 0;
+      }
+      epi_sync();
+      if (s_last == 1) {
+        __threadfence();
+        if (p.npref > 0) {
+          merge_staged(cur, j, first, last, et, n_et, watcher);
+        } else {
+          // (the 4-piece batches fit in the registers of the 4-copy layout only)
+          merge_job<D, R == 4 ? 4 : 1>(p, rowbits, cur, j, first, last, et, n_et);
         }
-        if (R > 1) epi_sync();  // the staging buffer is reused at the next piece
-          };
-    const int64_t x_end = in_piece ? e : b;
-    if (b < x_end) {
-      Job cur = job_at(p, gpre, b);
-      if (in_epi && !write_q(cur, false, 0u)) ok = false;
-      int pc = 0;
-      for (int64_t x0 = b; x0 < x_end; ++pc) {
-        const int n_in = (int)(min(e, cur.start + cur.n) - x0);
-        const bool more = x0 + n_in < e;
-        const Job nxt = more ? next_job(p, gpre, cur) : cur;
+      }
+      if (et == 0) p.ticket[j] = 0;
+      epi_sync();  // (the prefetch area and s_last are reused at the next piece)
+    };
+    if (in_piece && b < e) {
+      const PieceIter& it = s_it;
+      Job cur = it.j0;
+      int n_in = it.n0;
+      if (in_epi && !write_q(cur, false, 0u, [](uint64_t*, uint32_t) { return true; })) ok = false;
+      for (int pc = 0;; ++pc) {
+        Job nxt = cur;
+        int n_nxt = n_in;
+        const bool more = next_piece(p, gpre, it, pc + 1, nxt, n_nxt);
         if (side) {
           // one role per warp: the softmax warps run ahead into the next piece
           // while the epilogue warps finish this one
@@ -921,8 +1282,9 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
           run_groups(cur, n_in, pc);
           run_epilogue(cur, pc, more, nxt);
         }
-        x0 += n_in;
+        if (!more) break;
         cur = nxt;
+        n_in = n_nxt;
       }
     }
   }
@@ -934,6 +1296,7 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
       flag(p.dev_status, RGD_DEV_WAIT_TIMEOUT);
       const int issued = s_issued;
       for (int g = max(0, issued - ns); g < issued; ++g) mbar_wait(&full_bar[g % ns], (g / ns) & 1);
+      if (s_pref_n > 0) mbar_wait(&pref_bar, (uint32_t)(s_pref_n - 1) & 1u);  // the last partner prefetch
     }
     if ((warp == kMmaWarp || warp == kPvWarp) && lane == 0) {
       uint64_t* md = &mma_done[warp - kMmaWarp];
@@ -944,100 +1307,6 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
   }
   tc_fence_after();
   if (warp == kMmaWarp) tmem_dealloc(tmem, kTmemCols);
-}
-
-// Merge of a split job's partials (one block per job): with piece c holding the
-// unnormalised o_c and (m_c, l_c) in log2 units,
-//   out = sum_c 2^(m_c - M) o_c / sum_c 2^(m_c - M) l_c,  M = max_c m_c,
-//   lse = ln 2 * (M + log2 sum_c 2^(m_c - M) l_c).
-// Jobs held by one block were finished by the attention kernel.
-constexpr int kMergeThreads = 256;
-
-template <int D>
-__global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnParams p) {
-  // launched as a programmatic dependent of the attention kernel: its launch
-  // overlaps that kernel's tail, and this wait returns once it has completed
-  // and its writes are visible
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-  const int j = blockIdx.x;
-  const int g = j / p.Hkv, h = j % p.Hkv;
-  const int32_t* gp = p.gpre_ws;
-  const int64_t T = (int64_t)p.Hkv * gp[p.G];
-  const int n = gp[g + 1] - gp[g];
-  if (n == 0) return;
-  const int Ceff = (int)min((int64_t)p.C, T);
-  const int64_t start = (int64_t)p.Hkv * gp[g] + (int64_t)h * n;
-  const int first = cta_of(start, T, Ceff), last = cta_of(start + n - 1, T, Ceff);
-  if (first == last) return;
-  const int nq = p.nq, gq = p.gq;
-  constexpr int kChunks = D / 4;
-  constexpr int kP = 4;  // pieces whose loads are issued together
-  for (int item = threadIdx.x; item < nq * kChunks; item += kMergeThreads) {
-    const int i = item / kChunks, c4 = item % kChunks;
-    const int r = g * p.rpg + i / gq, hq = h * gq + i % gq;
-    if (!row_on(p, r)) continue;
-    float M = -INFINITY, Ls = 0.f;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int c0 = first; c0 <= last; c0 += kP) {
-      float2 ml[kP];
-      float4 v[kP];
-#pragma unroll
-      for (int t = 0; t < kP; ++t) {
-        if (c0 + t <= last) {
-          const int64_t si = ((int64_t)(c0 + t) + j) * nq + i;
-          ml[t] = p.slot_ml[si];
-          v[t] = reinterpret_cast<const float4*>(p.slot_o + si * D)[c4];
-        } else {
-          ml[t] = make_float2(-INFINITY, 0.f);
-        }
-      }
-      // online merge: the running (M, L, acc) absorbs up to kP pieces at once
-      float Mn = M;
-#pragma unroll
-      for (int t = 0; t < kP; ++t)
-        if (ml[t].y != 0.f) Mn = fmaxf(Mn, ml[t].x);
-      if (Mn == -INFINITY) continue;
-      const float f = (M == -INFINITY) ? 0.f : exp2f(M - Mn);
-      Ls *= f;
-      acc.x *= f;
-      acc.y *= f;
-      acc.z *= f;
-      acc.w *= f;
-#pragma unroll
-      for (int t = 0; t < kP; ++t) {
-        if (ml[t].y == 0.f) continue;
-        const float w = exp2f(ml[t].x - Mn);
-        Ls += w * ml[t].y;
-        acc.x += w * v[t].x;
-        acc.y += w * v[t].y;
-        acc.z += w * v[t].z;
-        acc.w += w * v[t].w;
-      }
-      M = Mn;
-    }
-    const float iv = Ls > 0.f ? 1.f / Ls : 0.f;
-    uint2 pk;
-    pk.x = pack_bf16x2(acc.x * iv, acc.y * iv);
-    pk.y = pack_bf16x2(acc.z * iv, acc.w * iv);
-    reinterpret_cast<uint2*>(p.out + ((int64_t)r * p.Hq + hq) * D)[c4] = pk;
-    if (p.lse && c4 == 0) p.lse[(int64_t)r * p.Hq + hq] = Ls > 0.f ? (M + log2f(Ls)) * kLn2 : -INFINITY;
-  }
-}
-
-// The merge kernel follows the attention kernel as a programmatic dependent.
-template <int D>
-cudaError_t launch_merge(const AttnParams& p, int J, cudaStream_t st) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(J);
-  cfg.blockDim = dim3(kMergeThreads);
-  cfg.dynamicSmemBytes = 0;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, attn_merge_kernel<D>, p);
 }
 
 // ---------------------------------------------------------------------------
@@ -1082,9 +1351,9 @@ int device_sm_count() {
 }
 
 struct Plan {
-  int nq, nslots, C, J;
+  int nq, nslots, C, J, npref;
   SmemLayout smem;
-  size_t gpre_off, ml_off, o_off, total;
+  size_t ticket_off, ml_off, o_off, total;
 };
 
 int check_shape(const rgd_attn_shape* s) {
@@ -1100,7 +1369,8 @@ int check_shape(const rgd_attn_shape* s) {
   RGD_CHECK_ARG((int64_t)s->num_pages * s->num_kv_heads * kPage < (int64_t)1 << 31,
                 "num_pages * num_kv_heads * page_size must be < 2^31");
   RGD_CHECK_ARG(s->max_prompt_pages >= 1 && s->max_suffix_pages >= 1, "block tables need >= 1 column");
-  RGD_CHECK_ARG(s->num_ctas >= 0 && s->reserved == 0, "num_ctas must be >= 0 and reserved 0");
+  RGD_CHECK_ARG(s->num_ctas >= 0 && s->num_ctas <= 65535 && s->reserved == 0,
+                "num_ctas must be in [0, 65535] and reserved 0");
   RGD_CHECK_ARG((int64_t)s->num_groups * (s->max_prompt_pages + (int64_t)s->rows_per_group * s->max_suffix_pages) *
                         s->num_kv_heads <
                     ((int64_t)1 << 31),
@@ -1119,21 +1389,34 @@ int make_plan(const rgd_attn_shape* s, Plan* pl) {
   pl->J = s->num_groups * s->num_kv_heads;
   // The ring holds at least three page groups: a group's slot is released by
   // its PV, which is issued after the next group's QK.
-  pl->nslots = kMaxSlots;
-  for (;;) {
-    const int R = s->num_groups * s->rows_per_group;
-    pl->smem = s->head_dim == 128 ? smem_layout<128>(pl->nslots, s->num_groups, R)
-                                  : smem_layout<64>(pl->nslots, s->num_groups, R);
-    if (pl->smem.total <= kSmemLimit) break;
-    if (pl->nslots <= 3)
-      return set_error(RGD_ERR_UNSUPPORTED, "shape needs more shared memory than an SM has (too many groups?)");
-    --pl->nslots;
+  // The shared memory holds the ring and, for the merge of a split job, up to
+  // two partner partials (a job spans at most three blocks when blocks hold
+  // about as many pages as a job).  Staging both partials is worth a ring slot
+  // (it keeps the merges of three-piece jobs off the end of the blocks), down
+  // to four slots; below that the ring comes first.
+  const int rows = s->num_groups * s->rows_per_group;
+  auto layout = [&](int nslots, int npref) {
+    return s->head_dim == 128 ? smem_layout<128>(nslots, s->num_groups, rows, pl->nq, npref)
+                              : smem_layout<64>(nslots, s->num_groups, rows, pl->nq, npref);
+  };
+  pl->nslots = 0;
+  for (int npref = 2; npref >= 0 && pl->nslots == 0; --npref) {
+    for (int ns = kMaxSlots; ns >= (npref > 0 ? 4 : 3); --ns) {
+      if (layout(ns, npref).total <= kSmemLimit) {
+        pl->nslots = ns;
+        pl->npref = npref;
+        break;
+      }
+    }
   }
+  if (pl->nslots == 0)
+    return set_error(RGD_ERR_UNSUPPORTED, "shape needs more shared memory than an SM has (too many groups?)");
+  pl->smem = layout(pl->nslots, pl->npref);
   auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
   const size_t n_part = (size_t)pl->C + pl->J - 1;  // partial-result slots
-  pl->gpre_off = 0;
-  pl->ml_off = up((size_t)(s->num_groups + 1) * sizeof(int32_t));
-  pl->o_off = pl->ml_off + up(n_part * pl->nq * sizeof(float2));
+  pl->ticket_off = 0;
+  pl->ml_off = up((size_t)pl->J * sizeof(int32_t));
+  pl->o_off = pl->ml_off + up(n_part * ml_stride(pl->nq) * sizeof(float2));
   pl->total = pl->o_off + up(n_part * pl->nq * s->head_dim * sizeof(float));
   return RGD_OK;
 }
@@ -1159,7 +1442,7 @@ extern "C" size_t rgd_prefix_decode_attn_workspace_size(const rgd_attn_shape* sh
 namespace rgd {
 namespace {
 
-// The attention kernel for one (head dim, copy count), then the split-job merge.
+// The attention kernel for one (head dim, copy count).
 template <int D, int R>
 int launch_attn(const CUtensorMap& tmK, const CUtensorMap& tmV, const AttnParams& p, const Plan& pl,
                 cudaStream_t st) {
@@ -1167,7 +1450,6 @@ int launch_attn(const CUtensorMap& tmK, const CUtensorMap& tmV, const AttnParams
   if (int rc = ensure_smem(attn_tc_kernel<D, R>, kSmemLimit, &done)) return rc;
   attn_tc_kernel<D, R><<<pl.C, Roles<R>::kThreads, pl.smem.total, st>>>(tmK, tmV, p);
   if (cudaError_t e = cudaGetLastError(); e != cudaSuccess) return cuda_error(e, "attention launch");
-  if (cudaError_t e = launch_merge<D>(p, pl.J, st); e != cudaSuccess) return cuda_error(e, "merge launch");
   return RGD_OK;
 }
 
@@ -1208,7 +1490,7 @@ extern "C" int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf1
   p.out = reinterpret_cast<__nv_bfloat16*>(out);
   p.lse = lse;
   uint8_t* ws = static_cast<uint8_t*>(workspace);
-  p.gpre_ws = reinterpret_cast<int32_t*>(ws + pl.gpre_off);
+  p.ticket = reinterpret_cast<int32_t*>(ws + pl.ticket_off);
   p.slot_ml = reinterpret_cast<float2*>(ws + pl.ml_off);
   p.slot_o = reinterpret_cast<float*>(ws + pl.o_off);
   p.dev_status = dev_status;
@@ -1222,6 +1504,7 @@ extern "C" int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf1
   p.max_sp = s.max_suffix_pages;
   p.nq = pl.nq;
   p.nslots = pl.nslots;
+  p.npref = pl.npref;
   p.C = pl.C;
   p.scale_log2 = softmax_scale * kLog2e;
 
@@ -1293,8 +1576,8 @@ extern "C" int rgd_prefix_decode_attn_noalloc(const rgd_attn_shape* shape, const
     }
     scratch = g_scratch_ptr[dev];
   }
-  // the array keeps the previous call's contents; every value a call reads from
-  // it was written earlier in the same call, so nothing needs clearing
+  // the array is zero when the module is loaded (device variables without an
+  // initializer are zero-filled) and every call leaves its job counters at zero
   return rgd_prefix_decode_attn(shape, q, k_pages, v_pages, prompt_block_table, prompt_len, suffix_block_table,
                                 suffix_len, row_active, softmax_scale, out, lse, scratch, kStaticScratchBytes,
                                 dev_status, stream);

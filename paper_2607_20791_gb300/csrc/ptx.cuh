@@ -58,6 +58,19 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Non-blocking test: has the phase with the given parity completed?
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 // As mbar_try_wait, but the thread may sleep up to `hint_ns` inside the
 // instruction (it wakes as soon as the phase completes), so that waiting warps
 // take no issue slots from working ones.
@@ -110,6 +123,21 @@ __device__ __forceinline__ void tma_load_3d_hint(void* dst, const CUtensorMap* m
       " [%0], [%1, {%3, %4, %5}], [%2], %6;"
       ::"r"(smem_u32(dst)), "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y), "r"(z), "l"(policy)
       : "memory");
+}
+
+// Acquire / release accesses (generic addresses).
+__device__ __forceinline__ int32_t ld_acquire_gpu(const int32_t* ptr) {
+  int32_t v;
+  asm volatile("ld.acquire.gpu.b32 %0, [%1];" : "=r"(v) : "l"(ptr) : "memory");
+  return v;
+}
+__device__ __forceinline__ int32_t ld_acquire_cta(const int32_t* ptr) {
+  int32_t v;
+  asm volatile("ld.acquire.cta.b32 %0, [%1];" : "=r"(v) : "l"(ptr) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release_cta(int32_t* ptr, int32_t v) {
+  asm volatile("st.release.cta.b32 [%0], %1;" ::"l"(ptr), "r"(v) : "memory");
 }
 
 __device__ __forceinline__ uint64_t policy_evict_first() {
@@ -201,6 +229,12 @@ __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 // Generic-proxy shared-memory writes made visible to the async proxy (TMA, MMA).
+// Orders this thread's generic-proxy view of global memory before its later
+// async-proxy (bulk copy) reads of it.
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
