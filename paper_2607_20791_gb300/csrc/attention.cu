@@ -124,7 +124,7 @@ struct AttnParams {
 // Shared-memory carve-up (identical on host and device).  The ring is 1024-byte
 // aligned: the 128-byte swizzle repeats every 8 rows of 128 bytes.
 struct SmemLayout {
-  int ring, red, gpre, gact, desc, rowbits, pref, total;
+  int ring, red, gpre, plen, desc, rowbits, slen, pref, total;
 };
 
 // Partial (m, l) pairs are stored nq rounded up to even per piece, so that
@@ -156,10 +156,11 @@ __host__ __device__ inline SmemLayout smem_layout(int nslots, int G, int R, int 
   // row-max exchange (2 buffers), row sums and running maxima of 2 pieces, O
   // staging for the copies >= 1 (2 buffers of at most 3 warps x 16 columns x 32 lanes)
   L.gpre = L.red + (2 * 4 * kRows + 2 * 4 * kRows + 2 * kRows + 2 * 3 * 4 * 32 * 4) * 4;
-  L.gact = align_up(L.gpre + (G + 1) * 4, 16);
-  L.desc = align_up(L.gact + G * 4, 16);
+  L.plen = align_up(L.gpre + (G + 1) * 4, 16);  // prompt length per group (clamped)
+  L.desc = align_up(L.plen + G * 4, 16);
   L.rowbits = align_up(L.desc + nslots * kGroupPages * 4, 16);  // one bit per row: active
-  L.pref = align_up(L.rowbits + (R + 31) / 32 * 4, 16);
+  L.slen = align_up(L.rowbits + (R + 31) / 32 * 4, 16);          // suffix length per row (0: inactive)
+  L.pref = align_up(L.slen + R * 4, 16);
   L.total = L.pref + npref * pref_bytes<D>(nq) + 1024;  // + slack for the 1024-byte aligned base
   return L;
 }
@@ -435,29 +436,41 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
     tmem_relinquish();
   }
   // ---- page counts per group and their exclusive prefix sum (every block) ----
-  // Rows are read in parallel (one global-memory latency, not one per row).
-  int32_t* gact = reinterpret_cast<int32_t*>(smem + L.gact);
-  for (int g = tid; g < p.G; g += kAttnThreads) {
-    gpre[g + 1] = 0;
-    gact[g] = 0;
+  // The lengths and activity flags are read once, all loads issued together
+  // (one global-memory latency), and kept in shared memory for the producer.
+  int32_t* plen_s = reinterpret_cast<int32_t*>(smem + L.plen);
+  int32_t* slen_s = reinterpret_cast<int32_t*>(smem + L.slen);
+  const int nrows = p.G * p.rpg;
+  for (int r0 = warp * 32; r0 < nrows; r0 += kAttnThreads) {  // (whole warps: the ballot below)
+    const int r = r0 + lane;
+    int act = 0, sl = 0;
+    if (r < nrows) {
+      act = p.row_active == nullptr ? 1 : p.row_active[r];
+      sl = p.suffix_len[r];
+      if (c == 0 && (sl < 0 || sl > p.max_sp * kPage)) flag(p.dev_status, RGD_DEV_BAD_PAGE);
+      slen_s[r] = act ? clamp_len(sl, p.max_sp) : 0;
+    }
+    const uint32_t bits = __ballot_sync(0xffffffffu, r < nrows && act != 0);
+    if (lane == 0) rowbits[r0 >> 5] = bits;
   }
-  for (int i = tid; i < (p.G * p.rpg + 31) / 32; i += kAttnThreads) rowbits[i] = 0;
+  for (int g = tid; g < p.G; g += kAttnThreads) {
+    const int pl = p.prompt_len[g];
+    if (c == 0 && (pl < 0 || pl > p.max_pp * kPage)) flag(p.dev_status, RGD_DEV_BAD_PAGE);
+    plen_s[g] = clamp_len(pl, p.max_pp);
+  }
   if (tid == 0) gpre[0] = 0;
   __syncthreads();
-  for (int r = tid; r < p.G * p.rpg; r += kAttnThreads) {
-    if (!row_on(p, r)) continue;
-    atomicAdd(&gpre[r / p.rpg + 1], (clamp_len(p.suffix_len[r], p.max_sp) + kPage - 1) / kPage);
-    atomicOr(&gact[r / p.rpg], 1);
-    atomicOr(&rowbits[r >> 5], 1u << (r & 31));
-  }
-  __syncthreads();
-  for (int g = tid; g < p.G; g += kAttnThreads)
-    gpre[g + 1] = gact[g] ? gpre[g + 1] + (clamp_len(p.prompt_len[g], p.max_pp) + kPage - 1) / kPage : 0;
-  if (c == 0) {
-    for (int g = tid; g < p.G; g += kAttnThreads)
-      if (p.prompt_len[g] < 0 || p.prompt_len[g] > p.max_pp * kPage) flag(p.dev_status, RGD_DEV_BAD_PAGE);
-    for (int r = tid; r < p.G * p.rpg; r += kAttnThreads)
-      if (p.suffix_len[r] < 0 || p.suffix_len[r] > p.max_sp * kPage) flag(p.dev_status, RGD_DEV_BAD_PAGE);
+  // a group's pages: its prompt pages if any row of it is active, plus its
+  // active rows' suffix pages
+  for (int g = tid; g < p.G; g += kAttnThreads) {
+    int n = 0;
+    bool any = false;
+    for (int rr = 0; rr < p.rpg; ++rr) {
+      const int r = g * p.rpg + rr;
+      n += (slen_s[r] + kPage - 1) / kPage;
+      any = any || ((rowbits[r >> 5] >> (r & 31)) & 1u);
+    }
+    gpre[g + 1] = any ? n + (plen_s[g] + kPage - 1) / kPage : 0;
   }
   tc_fence_before();
   __syncthreads();
@@ -543,7 +556,7 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
           ng = min(kGroupPages, npiece - (kin - jpos));
           if (mine) {
             const int k = (int)(x - jb.start);
-            const int plen = clamp_len(p.prompt_len[jb.g], p.max_pp);
+            const int plen = plen_s[jb.g];
             const int ppg = (plen + kPage - 1) / kPage;
             hh = jb.h;
             if (k < ppg) {
@@ -553,7 +566,7 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
               int ks = k - ppg;
               for (int rr = 0; rr < p.rpg; ++rr) {  // the active row holding suffix page ks
                 const int r = jb.g * p.rpg + rr;
-                const int slen = row_on(p, r) ? clamp_len(p.suffix_len[r], p.max_sp) : 0;
+                const int slen = slen_s[r];
                 const int np = (slen + kPage - 1) / kPage;
                 if (ks < np) {
                   page = __ldg(p.suffix_bt + (int64_t)r * p.max_sp + ks);
