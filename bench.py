@@ -18,7 +18,6 @@ every rank runs its own batch (weak scaling, no collective in the data path).
 from __future__ import annotations
 
 import argparse
-import inspect
 import hashlib
 import json
 import os
@@ -272,71 +271,63 @@ def run_ours(args):
         binding.rgd_probe_gate(trie, G, rpg, head.token_out, 1, rpg, case.gate.eos, case.gate.max_len, gstate,
                                gate_active, head.dev_status, stream=stream.cuda_stream)
 
-    # The whole step is one CUDA graph; a timing event recorded inside it (an
-    # "external" event) splits it into attention and sample head + gate.
-    one_graph = "external" in inspect.signature(torch.cuda.Event.__new__).parameters
+    # The whole step is one CUDA graph (the headline is timed on it).  The split
+    # into attention and sample head + gate comes from a second pass of the same
+    # steps launched eagerly, with events around each part: an event recorded
+    # inside the graph would itself leave the GPU idle for ~5 us per step.
     with torch.cuda.stream(stream):
         for _ in range(3):  # eager warm-up (also sets kernel attributes before capture)
             attn_call()
             head_gate_call()
         torch.cuda.synchronize()
-        if one_graph:
-            ev_mid = torch.cuda.Event(enable_timing=True, external=True)
-            g_step = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g_step, stream=stream):
-                attn_call()
-                ev_mid.record(stream)
-                head_gate_call()
-            graphs = [g_step]
-        else:
-            g_attn, g_hg = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g_attn, stream=stream):
-                attn_call()
-            with torch.cuda.graph(g_hg, stream=stream):
-                head_gate_call()
-            graphs = [g_attn, g_hg]
+        g_step = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_step, stream=stream):
+            attn_call()
+            head_gate_call()
         torch.cuda.synchronize()
     launches_per_step = 4  # attention (split jobs merged inside), sample head, gate-state reset, gate
 
     def one_step():
-        """Runs one timed step; returns (step, attention, head + gate) in ms."""
+        """Runs one timed step (the graph); returns its time in ms."""
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+        flush.fill_(1)
+        ev[0].record(stream)
+        g_step.replay()
+        ev[1].record(stream)
+        ev[1].synchronize()
+        return ev[0].elapsed_time(ev[1])
+
+    def split_step():
+        """Runs one step eagerly; returns (attention, head + gate) in ms."""
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
         flush.fill_(1)
         ev[0].record(stream)
-        if one_graph:
-            g_step.replay()
-            ev[2].record(stream)
-            ev[2].synchronize()  # ev_mid is re-recorded by every replay: read it now
-            mid = ev_mid
-        else:
-            g_attn.replay()
-            ev[1].record(stream)
-            g_hg.replay()
-            ev[2].record(stream)
-            ev[2].synchronize()
-            mid = ev[1]
-        return ev[0].elapsed_time(ev[2]), ev[0].elapsed_time(mid), mid.elapsed_time(ev[2])
+        attn_call()
+        ev[1].record(stream)
+        head_gate_call()
+        ev[2].record(stream)
+        ev[2].synchronize()
+        return ev[0].elapsed_time(ev[1]), ev[1].elapsed_time(ev[2])
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
             one_step()
+            split_step()
         torch.cuda.synchronize()
 
     if world > 1:
         import torch.distributed as dist
         dist.barrier()
     torch.cuda.synchronize()
-    times = []
     with ClockSampler(torch.cuda.current_device()) as clk:
         with torch.cuda.stream(stream):
-            for i in range(args.steps):
-                times.append(one_step())
+            step_ms = [one_step() for _ in range(args.steps)]
+            split = [split_step() for _ in range(args.steps)]
         torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
-    step_ms = [t[0] for t in times]
-    attn_ms = [t[1] for t in times]
-    hg_ms = [t[2] for t in times]
+    attn_ms = [t[0] for t in split]
+    hg_ms = [t[1] for t in split]
     mean_step = sum(step_ms) / len(step_ms)
     mean_attn = sum(attn_ms) / len(attn_ms)
     status = int(att.dev_status.item()) | int(head.dev_status.item())
@@ -371,8 +362,7 @@ def run_ours(args):
                 e2e_ev[i - args.warmup][0].record(stream)
             for k, t in pinned.items():
                 dst[k].copy_(t, non_blocking=True)
-            for g in graphs:
-                g.replay()
+            g_step.replay()
             tok_host.copy_(head.token_out, non_blocking=True)
             st_host.copy_(gstate, non_blocking=True)
             if i >= args.warmup:
@@ -402,9 +392,8 @@ def run_ours(args):
             "config": {"workload": WORKLOAD, "rows_per_step": rows_per_step, "groups": G,
                        "l2": "flushed between steps (256 MiB write, outside the timed events)",
                        "timing": "CUDA events per step on the launching stream around one CUDA graph of the "
-                                 "step (attention, sample head, gate), split by an event "
-                                 "recorded inside it" if one_graph else
-                                 "CUDA events per step around the attention graph and the sample-head/gate graph",
+                                 "step (attention, sample head, gate); kernels_ms and roofline from a second "
+                                 "pass of as many steps launched eagerly with events around each part",
                        "parallelism": f"replicas x{world}"},
             "step_hbm_gbs": step_gbs, "step_hbm_frac": step_gbs / peak,
             "step_algorithmic_bytes": step_bytes,
@@ -416,6 +405,7 @@ def run_ours(args):
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
                     "d2h_bytes_per_step": d2h_bytes, "ms_per_step": e2e_ms},
             "gpu_launches": launches_per_step * args.steps,
+            "split_pass_launches": launches_per_step * args.steps,
             "clocks": clocks, "dev_status": status,
         }
         print(json.dumps(line), flush=True)
