@@ -114,7 +114,7 @@ struct AttnParams {
   float* slot_o;    // [(C + J - 1) * nq, D]
   float2* slot_ml;  // [(C + J - 1) * ml_stride(nq)]
   int32_t* ticket;  // [J] pieces of a split job that have finished (zero between calls)
-  int npref;        // partner pieces whose partials fit the prefetch area (0..2)
+  int npref;        // partner pieces whose partials fit the prefetch area (1 or 2)
   int32_t* dev_status;
   int32_t G, rpg, Hq, Hkv, gq, num_pages, max_pp, max_sp;
   int32_t nq, nslots, C;
@@ -294,68 +294,6 @@ __device__ __forceinline__ bool wait_slot_gen(int32_t* gen, int32_t want, volati
       }
     }
     __nanosleep(32);
-  }
-}
-
-// Merge of split job jj's partials (pieces first..last, workspace slots
-// piece + jj) by n_threads threads, thread et taking items et, et + n_threads,
-// ... (item = 4 output columns of one query): with piece s holding the
-// unnormalised o_s and (m_s, l_s) in log2 units,
-//   out = sum_s 2^(m_s - M) o_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s.
-// kP pieces' loads are issued together (more registers, fewer round trips).
-template <int D, int kP>
-__device__ __forceinline__ void merge_job(const AttnParams& p, const uint32_t* rowbits, Job jb, int jj, int first,
-                                       int last, int et, int n_threads) {
-  constexpr int kC4 = D / 4;
-  const int nq = p.nq, gq = p.gq;
-  for (int item = et; item < nq * kC4; item += n_threads) {
-    const int i = item / kC4, c4 = item % kC4;
-    const int rr2 = jb.g * p.rpg + i / gq, hq2 = jb.h * gq + i % gq;
-    if (!((rowbits[rr2 >> 5] >> (rr2 & 31)) & 1u)) continue;
-    float Mm = -INFINITY, Lm = 0.f;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int c0 = first; c0 <= last; c0 += kP) {
-      float2 ml[kP];
-      float4 v[kP];
-#pragma unroll
-      for (int t = 0; t < kP; ++t) {
-        if (c0 + t <= last) {
-          const int64_t sl = (int64_t)(c0 + t) + jj;
-          ml[t] = __ldcg(p.slot_ml + sl * ml_stride(nq) + i);
-          v[t] = __ldcg(reinterpret_cast<const float4*>(p.slot_o + (sl * nq + i) * D) + c4);
-        } else {
-          ml[t] = make_float2(-INFINITY, 0.f);
-        }
-      }
-      float Mn = Mm;
-#pragma unroll
-      for (int t = 0; t < kP; ++t)
-        if (ml[t].y != 0.f) Mn = fmaxf(Mn, ml[t].x);
-      if (Mn == -INFINITY) continue;
-      const float f = (Mm == -INFINITY) ? 0.f : exp2f(Mm - Mn);
-      Lm *= f;
-      acc.x *= f;
-      acc.y *= f;
-      acc.z *= f;
-      acc.w *= f;
-#pragma unroll
-      for (int t = 0; t < kP; ++t) {
-        if (ml[t].y == 0.f) continue;
-        const float wt = exp2f(ml[t].x - Mn);
-        Lm += wt * ml[t].y;
-        acc.x += wt * v[t].x;
-        acc.y += wt * v[t].y;
-        acc.z += wt * v[t].z;
-        acc.w += wt * v[t].w;
-      }
-      Mm = Mn;
-    }
-    const float iv = Lm > 0.f ? 1.f / Lm : 0.f;
-    uint2 pk2;
-    pk2.x = pack_bf16x2(acc.x * iv, acc.y * iv);
-    pk2.y = pack_bf16x2(acc.z * iv, acc.w * iv);
-    reinterpret_cast<uint2*>(p.out + ((int64_t)rr2 * p.Hq + hq2) * D)[c4] = pk2;
-    if (p.lse && c4 == 0) p.lse[(int64_t)rr2 * p.Hq + hq2] = Lm > 0.f ? (Mm + log2f(Lm)) * kLn2 : -INFINITY;
   }
 }
 
@@ -1267,12 +1205,7 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
       epi_sync();
       if (s_last == 1) {
         __threadfence();
-        if (p.npref > 0) {
-          merge_staged(cur, j, first, last, et, n_et, watcher);
-        } else {
-          // (the 4-piece batches fit in the registers of the 4-copy layout only)
-          merge_job<D, R == 4 ? 4 : 1>(p, rowbits, cur, j, first, last, et, n_et);
-        }
+        merge_staged(cur, j, first, last, et, n_et, watcher);
       }
       if (et == 0) p.ticket[j] = 0;
       epi_sync();  // (the prefetch area and s_last are reused at the next piece)
@@ -1402,19 +1335,20 @@ int make_plan(const rgd_attn_shape* s, Plan* pl) {
   pl->J = s->num_groups * s->num_kv_heads;
   // The ring holds at least three page groups: a group's slot is released by
   // its PV, which is issued after the next group's QK.
-  // The shared memory holds the ring and, for the merge of a split job, up to
-  // two partner partials (a job spans at most three blocks when blocks hold
+  // The shared memory holds the ring and, for the merge of a split job, one
+  // or two partner partials (a job spans at most three blocks when blocks hold
   // about as many pages as a job).  Staging both partials is worth a ring slot
   // (it keeps the merges of three-piece jobs off the end of the blocks), down
-  // to four slots; below that the ring comes first.
+  // to four slots; one staged partial is the minimum (the merges go through
+  // that area).
   const int rows = s->num_groups * s->rows_per_group;
   auto layout = [&](int nslots, int npref) {
     return s->head_dim == 128 ? smem_layout<128>(nslots, s->num_groups, rows, pl->nq, npref)
                               : smem_layout<64>(nslots, s->num_groups, rows, pl->nq, npref);
   };
   pl->nslots = 0;
-  for (int npref = 2; npref >= 0 && pl->nslots == 0; --npref) {
-    for (int ns = kMaxSlots; ns >= (npref > 0 ? 4 : 3); --ns) {
+  for (int npref = 2; npref >= 1 && pl->nslots == 0; --npref) {
+    for (int ns = kMaxSlots; ns >= (npref > 1 ? 4 : 3); --ns) {
       if (layout(ns, npref).total <= kSmemLimit) {
         pl->nslots = ns;
         pl->npref = npref;
