@@ -133,11 +133,11 @@ struct Shared {
   float stripe_sum[kHeadWarps][kMaxStripes];
   float stripe_max[kHeadWarps][kMaxStripes];
   uint8_t stripe_list[kHeadWarps][kMaxStripes];  // pass 2: the stripes a warp re-reads
-  // published to the cluster
-  float cta_max;
-  int32_t cta_arg;
-  float cta_sum;
-  int32_t cta_cnt;
+  // pushed by every CTA of the cluster into every CTA's copy (slot = rank)
+  float cta_max[kClusterCtas];
+  int32_t cta_arg[kClusterCtas];
+  float cta_sum[kClusterCtas];
+  int32_t cta_cnt[kClusterCtas];
   // broadcast within the CTA
   float row_max;
   int32_t row_arg;
@@ -247,7 +247,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
     sh.red_i[warp] = bi;
   }
   __syncthreads();
-  if (tid == 0) {
+  if (warp == 0) {
     float v = sh.red_v[0];
     int32_t i = sh.red_i[0];
     for (int w = 1; w < kHeadWarps; ++w)
@@ -255,10 +255,17 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
         v = sh.red_v[w];
         i = sh.red_i[w];
       }
-    sh.cta_max = v;
-    sh.cta_arg = i;
+    // one lane per CTA of the cluster writes this CTA's maximum into that CTA
+    if (lane < kClusterCtas) {
+      Shared* o = cluster.map_shared_rank(&sh, lane);
+      o->cta_max[rank] = v;
+      o->cta_arg[rank] = i;
+    }
   }
-  cluster.sync();  // #1: range maxima visible to the cluster
+  // #1: every CTA's maximum is in every CTA's shared memory.  (All cluster
+  // traffic is writes before a barrier and local reads after it, so no CTA
+  // needs to outlive another's reads.)
+  cluster.sync();
   const float temp = p.temperature[row];
   const float mp = p.min_p[row];
   if (warp == 0) {
@@ -266,9 +273,8 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
     float v = -INFINITY;
     int32_t i = 0x7fffffff;
     if (lane < kClusterCtas) {
-      const Shared* o = cluster.map_shared_rank(&sh, lane);
-      v = o->cta_max;
-      i = o->cta_arg;
+      v = sh.cta_max[lane];
+      i = sh.cta_arg[lane];
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -304,7 +310,6 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
         if (p.kept_count) p.kept_count[row] = 1;
       }
     }
-    cluster.sync();  // keep this CTA's shared memory alive until every CTA has read it
     return;
   }
 
@@ -370,26 +375,28 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
     sh.red_c[warp] = cnt;
   }
   __syncthreads();
-  if (tid == 0) {
+  if (warp == 0) {
     KSum t;
     int32_t ct = 0;
     for (int w = 0; w < kHeadWarps; ++w) {
       t.add(sh.red_s[w]);
       ct += sh.red_c[w];
     }
-    sh.cta_sum = t.value();
-    sh.cta_cnt = ct;
+    if (lane < kClusterCtas) {
+      Shared* o = cluster.map_shared_rank(&sh, lane);
+      o->cta_sum[rank] = t.value();
+      o->cta_cnt[rank] = ct;
+    }
   }
-  cluster.sync();  // #2: range sums visible to the cluster
+  cluster.sync();  // #2: every CTA's sums are in every CTA's shared memory
 
   // ---- the draw: target u * Z; CTA, warp and stripe by prefix sums in index
   // order; then the stripe's lanes and the lane's elements --------------------
   float cs = 0.f;
   int32_t cc = 0;
   if (warp == 0 && lane < kClusterCtas) {
-    const Shared* o = cluster.map_shared_rank(&sh, lane);
-    cs = o->cta_sum;
-    cc = o->cta_cnt;
+    cs = sh.cta_sum[lane];
+    cc = sh.cta_cnt[lane];
   }
   if (warp == 0) {
 #pragma unroll
@@ -481,7 +488,6 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
       }
     }
   }
-  cluster.sync();  // #3: shared memory stays alive until the cluster is done reading it
 }
 
 }  // namespace
