@@ -197,8 +197,14 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
   // keep it, pass 2 (its last full read) lets it go
   const uint64_t keep_pol = policy_evict_last(), drop_pol = policy_evict_first();
   // the draw for this row, computed while the logits stream in
-  float u = 0.f;
+  // the row's parameters and the min-p offset T ln p_min (fp64 logarithm, one
+  // thread) before pass 1, off the path after the row maximum
+  const float temp = p.temperature[row];
+  const float mp = p.min_p[row];
+  const bool probe = p.is_probe && p.is_probe[row];
+  float u = 0.f, theta = -INFINITY;
   if (tid == 0) {
+    if (mp > 0.0f) theta = (float)((double)temp * log((double)mp));
     const uint64_t sd = p.seed[row];
     const uint32_t x0 = philox_word0((uint32_t)p.step, (uint32_t)(p.step >> 32), 0u, 0u, (uint32_t)sd,
                                      (uint32_t)(sd >> 32));
@@ -266,8 +272,6 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
   // traffic is writes before a barrier and local reads after it, so no CTA
   // needs to outlive another's reads.)
   cluster.sync();
-  const float temp = p.temperature[row];
-  const float mp = p.min_p[row];
   if (warp == 0) {
     // one lane per CTA of the cluster reads its maximum (the remote loads overlap)
     float v = -INFINITY;
@@ -288,15 +292,13 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
     if (lane == 0) {
       sh.row_max = v;
       sh.row_arg = i;
-      // the min-p cutoff fl32(M + fl32(T ln p_min)); the logarithm in fp64 by one thread
-      const float theta = (mp > 0.0f) ? (float)((double)temp * log((double)mp)) : -INFINITY;
-      sh.cut = __fadd_rn(v, theta);
+      sh.cut = __fadd_rn(v, theta);  // the min-p cutoff fl32(M + fl32(T ln p_min))
     }
   }
   __syncthreads();
   const float M = sh.row_max;
   const int32_t A = sh.row_arg;
-  const bool greedy = (p.is_probe && p.is_probe[row]) || temp == 0.0f;
+  const bool greedy = probe || temp == 0.0f;
   const bool bad = !(temp >= 0.0f) || !isfinite(temp) || !(mp >= 0.0f && mp <= 1.0f) || !isfinite(M) ||
                    A >= p.vocab;
   if (greedy || bad) {
