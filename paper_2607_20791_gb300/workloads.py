@@ -409,6 +409,46 @@ def gate_sweep(groups: int = 1024, n_seq: int = 1000, vocab: int = 128256, n_ste
                     max_len=n_steps, rows_per_group=1)
 
 
+@dataclasses.dataclass
+class PrecheckCase:
+    """Inputs of the residual-stream precheck (App. A): one last-prompt-token
+    activation per group, a logistic readout (w, b) and the skip threshold."""
+    name: str
+    h: np.ndarray        # float32 [G, d] or uint16 bf16 bits [G, d]
+    dtype: str           # "f32" or "bf16"
+    w: np.ndarray        # float32 [d]
+    b: float
+    theta: float
+    rows_per_group: int
+
+    @property
+    def groups(self) -> int:
+        return self.h.shape[0]
+
+    @property
+    def d(self) -> int:
+        return self.h.shape[1]
+
+
+def make_precheck_case(name: str, groups: int, d: int, dtype: str, theta: float, seed: int,
+                       weight_scale: float = 1.0, bias: float = 0.0, rows_per_group: int = 5) -> PrecheckCase:
+    """Activations ~ N(0, 1) (fp32, or rounded to bf16), weights ~ N(0, weight_scale^2 / d)
+    in fp32, so that the readout's spread across groups is about weight_scale."""
+    h32 = _rng(seed, 41).standard_normal((groups, d), dtype=np.float32)
+    h = h32 if dtype == "f32" else f32_to_bf16_bits(h32)
+    w = (_rng(seed, 42).standard_normal(d) * (weight_scale / np.sqrt(d))).astype(np.float32)
+    return PrecheckCase(name=name, h=h, dtype=dtype, w=w, b=float(bias), theta=float(theta),
+                        rows_per_group=rows_per_group)
+
+
+def llama8b_precheck(seed: int = 0) -> PrecheckCase:
+    """The Llama-3-8B-shaped step's 16 prompt groups: d = 4096 bf16 activations,
+    the paper's calibrated Llama threshold theta = 1e-5, a readout spread of 8 so
+    that a few groups fall under it."""
+    return make_precheck_case("llama8b_precheck", 16, 4096, "bf16", 1e-5, seed, weight_scale=8.0,
+                              bias=-2.0, rows_per_group=5)
+
+
 CONFIGS = {
     "tiny": tiny,
     "llama8b": llama8b,
