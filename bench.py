@@ -332,6 +332,28 @@ def run_ours(args):
     mean_attn = sum(attn_ms) / len(attn_ms)
     status = int(att.dev_status.item()) | int(head.dev_status.item())
 
+    # ---- the residual-stream precheck (App. A): once per prompt, not per step;
+    # timed alone on the step's 16 groups (d = 4096 bf16), L2 flushed before each
+    pre = workloads.llama8b_precheck(seed=rank)
+    pre_h = torch.from_numpy(pre.h.view(np.int16)).to(dev).view(torch.bfloat16)
+    pre_w = torch.from_numpy(pre.w).to(dev)
+    pre_st = binding.new_gate_state(G, device=dev)
+    pre_prob = torch.empty(G, dtype=torch.float32, device=dev)
+    pre_ms = []
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup + args.steps):
+            binding.rgd_gate_state_init(pre_st, G, stream=stream.cuda_stream)
+            flush.fill_(1)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            binding.rgd_residual_precheck(pre_h, pre_w, pre.b, pre.theta, rpg, pre_st, None, pre_prob,
+                                          stream=stream.cuda_stream)
+            e1.record(stream)
+            e1.synchronize()
+            if i >= args.warmup:
+                pre_ms.append(e0.elapsed_time(e1))
+    pre_bytes = pre.groups * pre.d * 2 + pre.d * 4 + pre.groups * (4 + 20)
+
     # ---- end to end through the public API with host buffers ----------------
     h2d_src = {
         "q": case.attn.q, "logits": case.head.logits, "prompt_block_table": case.attn.prompt_block_table,
@@ -406,6 +428,9 @@ def run_ours(args):
                     "d2h_bytes_per_step": d2h_bytes, "ms_per_step": e2e_ms},
             "gpu_launches": launches_per_step * args.steps,
             "split_pass_launches": launches_per_step * args.steps,
+            "residual_precheck": {"us": 1e3 * sorted(pre_ms)[len(pre_ms) // 2], "groups": pre.groups, "d": pre.d,
+                                  "bytes": pre_bytes, "bound": "launch latency (a d + 1 logistic readout)",
+                                  "note": "once per prompt, outside the step"},
             "clocks": clocks, "dev_status": status,
         }
         print(json.dumps(line), flush=True)

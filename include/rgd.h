@@ -13,7 +13,9 @@
  * This library implements one decode step of that loop as CUDA kernels:
  *   rgd_prefix_decode_attn  shared-prefix split-KV decode attention,
  *   rgd_sample_head         greedy argmax / temperature + min-p + Philox sample,
- *   rgd_probe_gate          per-token refusal-prefix gate on a token trie.
+ *   rgd_probe_gate          per-token refusal-prefix gate on a token trie,
+ *   rgd_residual_precheck   the residual-stream classifier that lets a prompt
+ *                           skip the probe (App. A), once per prompt.
  *
  * Conventions for every entry point
  *   - Tensor pointers are DEVICE pointers owned by the caller unless a comment
@@ -249,6 +251,31 @@ int rgd_probe_gate(const rgd_trie* trie, int32_t groups, int32_t rows_per_group,
                    const int32_t* probe_tokens, int32_t n_tokens, int64_t token_stride,
                    int32_t eos_token, int32_t max_len, rgd_gate_state* state,
                    uint8_t* row_active, int32_t* dev_status, rgd_stream_t stream);
+
+/* ------------------------------------------------------------------------ */
+/* Residual-stream precheck (App. A)                                          */
+/* ------------------------------------------------------------------------ */
+
+/* Logistic readout of each group's last-prompt-token activation, run once
+ * before the probe's first token:
+ *   z_g = sum_i w[i] * h[g, i] + bias,  p_g = 1 / (1 + exp(-z_g)),
+ * and a group with p_g <= theta skips the greedy probe (App. A: the prompt
+ * decodes directly at high temperature).  For such a group whose state is
+ * still the fresh empty probe (pending, no token consumed), the state becomes
+ * decision RGD_NON_REFUSAL, done = 1, decisive_step -1 (decided before any
+ * probe token), and its probe row (row g * rows_per_group) is cleared in
+ * row_active; the sample rows stay on.  Other groups are left unchanged.
+ *   h           device, [groups, d], dtype RGD_F32 or RGD_BF16, row-major
+ *   w           device float [d]; bias, theta in [0, 1] by value
+ *   prob_out    device float [groups] (p_g) or NULL
+ *   state       device rgd_gate_state [groups]; row_active device
+ *               uint8 [groups * rows_per_group] or NULL
+ * z is accumulated in fp32 (the decision can differ from exact arithmetic
+ * only when z is within the fp32 rounding of its sum from the threshold's
+ * logit).  One kernel on `stream`, one block per group. */
+int rgd_residual_precheck(int32_t groups, int32_t d, int32_t dtype, const void* h, const float* w, float bias,
+                          float theta, int32_t rows_per_group, float* prob_out, rgd_gate_state* state,
+                          uint8_t* row_active, int32_t* dev_status, rgd_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -62,6 +62,7 @@ _SIGNATURES = {
     "rgd_trie_info": (ctypes.c_int, [_P, ctypes.POINTER(_I32), ctypes.POINTER(_I32)]),
     "rgd_gate_state_init": (ctypes.c_int, [_P, _I32, _P]),
     "rgd_probe_gate": (ctypes.c_int, [_P, _I32, _I32, _P, _I32, _I64, _I32, _I32, _P, _P, _P, _P]),
+    "rgd_residual_precheck": (ctypes.c_int, [_I32, _I32, _I32, _P, _P, _F, _F, _I32, _P, _P, _P, _P, _P]),
 }
 
 
@@ -234,6 +235,22 @@ def rgd_probe_gate(trie: Trie, groups: int, rows_per_group: int, probe_tokens, n
     _check(load_library().rgd_probe_gate(
         trie.handle, int(groups), int(rows_per_group), _ptr(probe_tokens, "probe_tokens", torch.int32),
         int(n_tokens), int(token_stride), int(eos_token), int(max_len), _ptr(state, "state"),
+        _ptr(row_active, "row_active", torch.uint8, optional=True),
+        _ptr(dev_status, "dev_status", torch.int32, optional=True), _stream(stream)))
+
+
+def rgd_residual_precheck(h, w, bias: float, theta: float, rows_per_group: int, state, row_active=None,
+                          prob_out=None, dev_status=None, stream=None) -> None:
+    import torch
+    if h.dim() != 2:
+        raise ValueError("h must be [groups, d]")
+    dtype = {torch.float32: RGD_F32, torch.bfloat16: RGD_BF16}.get(h.dtype)
+    if dtype is None:
+        raise TypeError("h must be float32 or bfloat16")
+    groups, d = h.shape
+    _check(load_library().rgd_residual_precheck(
+        int(groups), int(d), dtype, _ptr(h, "h"), _ptr(w, "w", torch.float32), float(bias), float(theta),
+        int(rows_per_group), _ptr(prob_out, "prob_out", torch.float32, optional=True), _ptr(state, "state"),
         _ptr(row_active, "row_active", torch.uint8, optional=True),
         _ptr(dev_status, "dev_status", torch.int32, optional=True), _stream(stream)))
 

@@ -45,6 +45,14 @@ def test_version_and_argument_errors_without_gpu(lib_path):
     assert rc == binding.RGD_ERR_INVALID_ARG
     rc = lib.rgd_probe_gate(None, 1, 1, None, 1, 1, -1, 4, None, None, None, None)
     assert rc == binding.RGD_ERR_INVALID_ARG
+    # the residual precheck: theta outside [0, 1], a bad dtype, missing tensors
+    for theta, dtype in ((1.5, 0), (-0.1, 0), (0.5, 7)):
+        rc = lib.rgd_residual_precheck(4, 16, dtype, 1, 1, 0.0, theta, 5, None, 1, None, None, None)
+        assert rc == binding.RGD_ERR_INVALID_ARG, (theta, dtype)
+    assert b"theta" in lib.rgd_last_error_string() or b"dtype" in lib.rgd_last_error_string()
+    rc = lib.rgd_residual_precheck(4, 16, 0, None, None, 0.0, 0.5, 5, None, None, None, None, None)
+    assert rc == binding.RGD_ERR_INVALID_ARG
+    assert lib.rgd_residual_precheck(0, 16, 0, None, None, 0.0, 0.5, 5, None, None, None, None, None) == 0
 
 
 def test_workspace_size_grows_with_blocks(lib_path):
@@ -54,7 +62,7 @@ def test_workspace_size_grows_with_blocks(lib_path):
     a = lib.rgd_prefix_decode_attn_workspace_size(ctypes.byref(s))
     s.num_ctas = 400
     b = lib.rgd_prefix_decode_attn_workspace_size(ctypes.byref(s))
-    # the page-count prefix of 16 groups + (ctas + jobs - 1) partial slots of 20 queries x (128 + 2) floats
+    # one ticket per job + (ctas + jobs - 1) partial slots of 20 queries x (128 + 2) floats
     grow = 300 * 20 * 128 * 4 + 300 * 20 * 8
     assert grow <= b - a < grow + 512  # each region is padded to 256 bytes
     s.reserved = 1
