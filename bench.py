@@ -354,6 +354,26 @@ def run_ours(args):
                 pre_ms.append(e0.elapsed_time(e1))
     pre_bytes = pre.groups * pre.d * 2 + pre.d * 4 + pre.groups * (4 + 20)
 
+    # ---- the soft compatibility gate (the appendix ablation's Alg. 2): an
+    # alternative to the hard gate; timed alone on the step's probe rows from a
+    # fresh state (top-K 40, rho 0.1; the step's greedy tokens mostly leave the
+    # refusal set, so the soft branch runs), L2 flushed before each call
+    soft_tok = torch.empty(G, dtype=torch.int32, device=dev)
+    soft_ms = []
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup + args.steps):
+            binding.rgd_gate_state_init(pre_st, G, stream=stream.cuda_stream)
+            flush.fill_(1)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            binding.rgd_soft_gate(trie, G, rpg, head.logits, rpg * head.logits.shape[1], 40, 0.1, 8,
+                                  case.gate.eos, case.gate.max_len, pre_st, soft_tok, stream=stream.cuda_stream)
+            e1.record(stream)
+            e1.synchronize()
+            if i >= args.warmup:
+                soft_ms.append(e0.elapsed_time(e1))
+    soft_bytes = G * head.logits.shape[1] * head.logits.element_size()
+
     # ---- end to end through the public API with host buffers ----------------
     h2d_src = {
         "q": case.attn.q, "logits": case.head.logits, "prompt_block_table": case.attn.prompt_block_table,
@@ -428,6 +448,9 @@ def run_ours(args):
                     "d2h_bytes_per_step": d2h_bytes, "ms_per_step": e2e_ms},
             "gpu_launches": launches_per_step * args.steps,
             "split_pass_launches": launches_per_step * args.steps,
+            "soft_gate": {"us": 1e3 * sorted(soft_ms)[len(soft_ms) // 2], "groups": G,
+                          "bytes": soft_bytes, "gbs": soft_bytes / (sorted(soft_ms)[len(soft_ms) // 2] / 1e3) / 1e9,
+                          "note": "alternative to the hard gate (top-K 40, rho 0.1), outside the step"},
             "residual_precheck": {"us": 1e3 * sorted(pre_ms)[len(pre_ms) // 2], "groups": pre.groups, "d": pre.d,
                                   "bytes": pre_bytes, "bound": "launch latency (a d + 1 logistic readout)",
                                   "note": "once per prompt, outside the step"},

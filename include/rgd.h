@@ -14,6 +14,7 @@
  *   rgd_prefix_decode_attn  shared-prefix split-KV decode attention,
  *   rgd_sample_head         greedy argmax / temperature + min-p + Philox sample,
  *   rgd_probe_gate          per-token refusal-prefix gate on a token trie,
+ *   rgd_soft_gate           its soft variant (the appendix ablation, Alg. 2),
  *   rgd_residual_precheck   the residual-stream classifier that lets a prompt
  *                           skip the probe (App. A), once per prompt.
  *
@@ -251,6 +252,32 @@ int rgd_probe_gate(const rgd_trie* trie, int32_t groups, int32_t rows_per_group,
                    const int32_t* probe_tokens, int32_t n_tokens, int64_t token_stride,
                    int32_t eos_token, int32_t max_len, rgd_gate_state* state,
                    uint8_t* row_active, int32_t* dev_status, rgd_stream_t stream);
+
+/* Soft compatibility gate (the appendix ablation's Alg. 2): one probe step per
+ * group from the probe row's logits.  With y the greedy token (argmax, lowest
+ * index on ties): after the first c probe steps, or when y is the stop token,
+ * or when q || y stays refusal-compatible, this is the hard gate's step with
+ * y.  Otherwise the top_k tokens of softmax(logits) (larger logit first, lower
+ * index first on ties) that keep q compatible -- the trie children of q's node,
+ * and the stop token, which does not change q -- form A_ref with mass m (their
+ * softmax probabilities summed); when A_ref is non-empty and m >= rho the most
+ * probable of them, a*, is appended instead of y (the caller feeds it back as
+ * the probe's token), else the probe is discarded: NON_REFUSAL at this step.
+ *   probe_logits   device [groups rows of row_stride elements]: group g's probe
+ *                  logits at probe_logits + g * row_stride (RGD_F32 / RGD_BF16);
+ *                  use the step's logits with row_stride = rows_per_group * vocab
+ *   token_out      device int32 [groups]: the token appended this step (y or
+ *                  a*), -1 when none (probe discarded or already ended)
+ *   mass_out       device float [groups] or NULL: m when the soft branch ran,
+ *                  else -1
+ * State and row_active as for rgd_probe_gate.  m is accumulated in fp32 (the
+ * decision can differ from exact arithmetic only when m is within ~1e-6
+ * relative of rho).  RGD_ERR_UNSUPPORTED when a trie node has more than 2047
+ * children.  One kernel on `stream`, one block per group. */
+int rgd_soft_gate(const rgd_trie* trie, int32_t groups, int32_t rows_per_group, int32_t vocab, int32_t dtype,
+                  const void* probe_logits, int64_t row_stride, int32_t top_k, float rho, int32_t c,
+                  int32_t eos_token, int32_t max_len, rgd_gate_state* state, uint8_t* row_active,
+                  int32_t* token_out, float* mass_out, int32_t* dev_status, rgd_stream_t stream);
 
 /* ------------------------------------------------------------------------ */
 /* Residual-stream precheck (App. A)                                          */

@@ -63,6 +63,8 @@ _SIGNATURES = {
     "rgd_gate_state_init": (ctypes.c_int, [_P, _I32, _P]),
     "rgd_probe_gate": (ctypes.c_int, [_P, _I32, _I32, _P, _I32, _I64, _I32, _I32, _P, _P, _P, _P]),
     "rgd_residual_precheck": (ctypes.c_int, [_I32, _I32, _I32, _P, _P, _F, _F, _I32, _P, _P, _P, _P, _P]),
+    "rgd_soft_gate": (ctypes.c_int, [_P, _I32, _I32, _I32, _I32, _P, _I64, _I32, _F, _I32, _I32, _I32, _P, _P,
+                                     _P, _P, _P, _P]),
 }
 
 
@@ -252,6 +254,24 @@ def rgd_residual_precheck(h, w, bias: float, theta: float, rows_per_group: int, 
         int(groups), int(d), dtype, _ptr(h, "h"), _ptr(w, "w", torch.float32), float(bias), float(theta),
         int(rows_per_group), _ptr(prob_out, "prob_out", torch.float32, optional=True), _ptr(state, "state"),
         _ptr(row_active, "row_active", torch.uint8, optional=True),
+        _ptr(dev_status, "dev_status", torch.int32, optional=True), _stream(stream)))
+
+
+def rgd_soft_gate(trie: Trie, groups: int, rows_per_group: int, logits, row_stride: int, top_k: int, rho: float,
+                  c: int, eos_token: int, max_len: int, state, token_out, row_active=None, mass_out=None,
+                  dev_status=None, stream=None) -> None:
+    """``logits`` is the step's [rows, vocab] tensor (or any tensor whose rows
+    g * row_stride / vocab hold group g's probe logits)."""
+    import torch
+    dtype = {torch.float32: RGD_F32, torch.bfloat16: RGD_BF16}.get(logits.dtype)
+    if dtype is None:
+        raise TypeError("logits must be float32 or bfloat16")
+    vocab = logits.shape[-1]
+    _check(load_library().rgd_soft_gate(
+        trie.handle, int(groups), int(rows_per_group), int(vocab), dtype, _ptr(logits, "logits"), int(row_stride),
+        int(top_k), float(rho), int(c), int(eos_token), int(max_len), _ptr(state, "state"),
+        _ptr(row_active, "row_active", torch.uint8, optional=True), _ptr(token_out, "token_out", torch.int32),
+        _ptr(mass_out, "mass_out", torch.float32, optional=True),
         _ptr(dev_status, "dev_status", torch.int32, optional=True), _stream(stream)))
 
 

@@ -9,6 +9,7 @@
 // predicate after every greedy probe token (the cap c does not change the
 // outcome of the hard gate).
 #include <algorithm>
+#include <cmath>
 #include <map>
 #include <vector>
 
@@ -22,6 +23,7 @@ struct rgd_trie {
   int32_t* child_tok = nullptr;    // [num_edges], sorted within a node
   int32_t* child_node = nullptr;   // [num_edges]
   uint8_t* confirm = nullptr;      // [num_nodes]: ends a prefix of length >= min_confirm
+  int32_t max_children = 0;        // the largest number of children of a node
   int device = 0;
 };
 
@@ -63,6 +65,60 @@ __global__ void gate_state_init_kernel(rgd_gate_state* st, int32_t groups) {
   st[g] = s;
 }
 
+// One probe token y (the stop token, or y >= 0) through the hard gate, for a
+// state whose probe has not ended.
+__device__ void consume_token(const TrieView& t, rgd_gate_state& s, int32_t y, int32_t eos, int32_t max_len,
+                              bool root_has_children) {
+  if (eos >= 0 && y == eos) {
+    const int32_t step = s.steps++;
+    s.done = 1;
+    if (s.decision == RGD_PENDING) {
+      // a pending probe is compatible, except the empty probe against an empty set
+      const bool ok = s.length > 0 || root_has_children;
+      s.decision = ok ? RGD_REFUSAL : RGD_NON_REFUSAL;
+      s.decisive_step = step;
+    }
+    return;
+  }
+  const int32_t step = s.steps++;
+  s.length++;
+  if (!s.confirmed) {
+    const int32_t e = find_child(t, s.node, y);
+    if (e < 0) {
+      s.decision = RGD_NON_REFUSAL;
+      s.decisive_step = step;
+      s.done = 1;
+      return;
+    }
+    s.node = __ldg(t.child_node + e);
+    if (__ldg(t.confirm + s.node)) {
+      s.confirmed = 1;
+      if (s.decision == RGD_PENDING) {
+        s.decision = RGD_REFUSAL;
+        s.decisive_step = step;
+      }
+    }
+  }
+  if (s.length >= max_len) {
+    s.done = 1;
+    if (s.decision == RGD_PENDING) {
+      s.decision = RGD_REFUSAL;
+      s.decisive_step = step;
+    }
+  }
+}
+
+// The gate's row mask: the probe row off once the probe has ended, the sample
+// rows off once the outcome is REFUSAL.
+__device__ __forceinline__ void mask_rows(const rgd_gate_state& s, uint8_t* row_active, int32_t g,
+                                          int32_t rows_per_group) {
+  if (!row_active) return;
+  uint8_t* ra = row_active + (int64_t)g * rows_per_group;
+  if (s.done) ra[0] = 0;
+  if (s.decision == RGD_REFUSAL)
+    for (int32_t i = 1; i < rows_per_group; ++i) ra[i] = 0;
+}
+
 __global__ void probe_gate_kernel(TrieView t, int32_t groups, int32_t rows_per_group,
                                   const int32_t* __restrict__ tokens, int32_t n_tokens, int64_t stride,
                                   int32_t eos, int32_t max_len, rgd_gate_state* __restrict__ state,
@@ -74,56 +130,246 @@ __global__ void probe_gate_kernel(TrieView t, int32_t groups, int32_t rows_per_g
   bool bad_token = false;
   for (int32_t k = 0; k < n_tokens && !s.done; ++k) {
     const int32_t y = __ldg(tokens + (int64_t)g * stride + k);
-    if (eos >= 0 && y == eos) {
-      const int32_t step = s.steps++;
-      s.done = 1;
-      if (s.decision == RGD_PENDING) {
-        // a pending probe is compatible, except the empty probe against an empty set
-        const bool ok = s.length > 0 || root_has_children;
-        s.decision = ok ? RGD_REFUSAL : RGD_NON_REFUSAL;
-        s.decisive_step = step;
-      }
-      break;
-    }
-    if (y < 0) {
+    if (y < 0 && !(eos >= 0 && y == eos)) {
       bad_token = true;
       continue;
     }
-    const int32_t step = s.steps++;
-    s.length++;
-    if (!s.confirmed) {
-      const int32_t e = find_child(t, s.node, y);
-      if (e < 0) {
-        s.decision = RGD_NON_REFUSAL;
-        s.decisive_step = step;
-        s.done = 1;
-        break;
-      }
-      s.node = __ldg(t.child_node + e);
-      if (__ldg(t.confirm + s.node)) {
-        s.confirmed = 1;
-        if (s.decision == RGD_PENDING) {
-          s.decision = RGD_REFUSAL;
-          s.decisive_step = step;
-        }
-      }
-    }
-    if (s.length >= max_len) {
-      s.done = 1;
-      if (s.decision == RGD_PENDING) {
-        s.decision = RGD_REFUSAL;
-        s.decisive_step = step;
-      }
-    }
+    consume_token(t, s, y, eos, max_len, root_has_children);
   }
   state[g] = s;
   if (bad_token && dev_status) atomicOr(dev_status, RGD_DEV_BAD_TOKEN);
-  if (row_active) {
-    uint8_t* ra = row_active + (int64_t)g * rows_per_group;
-    if (s.done) ra[0] = 0;
-    if (s.decision == RGD_REFUSAL)
-      for (int32_t i = 1; i < rows_per_group; ++i) ra[i] = 0;
+  mask_rows(s, row_active, g, rows_per_group);
+}
+
+// ---------------------------------------------------------------------------
+// Soft compatibility gate (the appendix ablation's Alg. 2), one probe step.
+// In the first c steps, a greedy token y that would leave the refusal-prefix
+// set does not end the probe at once: among the top-K tokens of the probe's
+// next-token distribution (softmax of its logits; ties to the lower index),
+// the refusal-compatible ones -- the children of the probe's trie node, and
+// the stop token, which d(q) drops -- are found, and if their probability
+// mass m reaches rho the most probable of them is appended instead.
+//
+// One block per group.  Pass 1 reads the probe's logits once: the maximum, its
+// lowest index (y) and the softmax normaliser Z (per-thread online sums).  The
+// soft branch then sorts the compatible candidates by logit in shared memory
+// (bitonic sort of (logit, token) keys) and counts, in passes over the logits
+// (from L2), how many tokens rank above each of the next 32 candidates; the
+// ranks grow along the sorted order, so the counting stops at the first
+// candidate outside the top K.
+constexpr int kSoftThreads = 512;
+constexpr int kMaxCand = 2048;  // a node's children + the stop token, sorted in shared memory
+constexpr int kChunk = 32;      // candidates ranked per pass over the logits
+
+struct SoftShared {
+  uint64_t key[kMaxCand];
+  float red_m[kSoftThreads / 32], red_z[kSoftThreads / 32];
+  int32_t red_i[kSoftThreads / 32];
+  int32_t cnt[kChunk];
+  float cv[kChunk];   // the chunk's candidates: logits and tokens
+  int32_t ci[kChunk];
+  rgd_gate_state s;
+  float M, Z, mass;
+  int32_t y, mode, ncand, n_in, stop;
+};
+
+template <typename LT>
+__device__ __forceinline__ float logit_at(const LT* row, int64_t i);
+template <>
+__device__ __forceinline__ float logit_at<float>(const float* row, int64_t i) {
+  return __ldg(row + i);
+}
+template <>
+__device__ __forceinline__ float logit_at<uint16_t>(const uint16_t* row, int64_t i) {
+  return __uint_as_float((uint32_t)__ldg(row + i) << 16);
+}
+
+// Order-preserving key: ascending keys = logits descending, then tokens ascending.
+__device__ __forceinline__ uint64_t rank_key(float v, int32_t tok) {
+  uint32_t u = __float_as_uint(v);
+  u = (u & 0x80000000u) ? ~u : (u | 0x80000000u);  // ascending with v
+  return ((uint64_t)(~u) << 32) | (uint32_t)tok;
+}
+__device__ __forceinline__ float key_logit(uint64_t k) {
+  uint32_t u = ~(uint32_t)(k >> 32);
+  u = (u & 0x80000000u) ? (u & 0x7fffffffu) : ~u;
+  return __uint_as_float(u);
+}
+
+// (v, i) ranks above (w, j): a larger logit, or the same logit and a lower index.
+__device__ __forceinline__ bool above(float v, int64_t i, float w, int64_t j) { return v > w || (v == w && i < j); }
+
+template <typename LT>
+__global__ void __launch_bounds__(kSoftThreads)
+    soft_gate_kernel(TrieView t, int32_t rows_per_group, int32_t vocab, const LT* __restrict__ logits,
+                     int64_t row_stride, int32_t top_k, float rho, int32_t c, int32_t eos, int32_t max_len,
+                     rgd_gate_state* __restrict__ state, uint8_t* __restrict__ row_active, int32_t* token_out,
+                     float* mass_out) {
+  __shared__ SoftShared sh;
+  const int g = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const LT* row = logits + (int64_t)g * row_stride;
+  if (tid == 0) {
+    sh.s = state[g];
+    sh.mode = 0;
+    sh.mass = -1.f;
   }
+  __syncthreads();
+  if (sh.s.done) {  // (uniform) nothing to consume
+    if (tid == 0) {
+      token_out[g] = -1;
+      if (mass_out) mass_out[g] = -1.f;
+    }
+    return;
+  }
+  // ---- pass 1: maximum, its lowest index, and Z = sum exp(l - max) ----
+  float m = -INFINITY, z = 0.f;
+  int32_t mi = 0x7fffffff;
+#pragma unroll 8
+  for (int32_t i = tid; i < vocab; i += kSoftThreads) {
+    const float v = logit_at<LT>(row, i);
+    if (v > m) {  // indices grow along a thread: strict > keeps the lowest
+      z = (m == -INFINITY) ? 1.f : z * expf(m - v) + 1.f;
+      m = v;
+      mi = i;
+    } else if (m != -INFINITY) {  // (with m = -inf, v is -inf too and adds nothing)
+      z += expf(v - m);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float om = __shfl_xor_sync(0xffffffffu, m, o), oz = __shfl_xor_sync(0xffffffffu, z, o);
+    const int32_t oi = __shfl_xor_sync(0xffffffffu, mi, o);
+    const float nm = fmaxf(m, om);
+    z = (m == -INFINITY ? 0.f : z * expf(m - nm)) + (om == -INFINITY ? 0.f : oz * expf(om - nm));
+    if (om > m || (om == m && oi < mi)) mi = oi;
+    m = nm;
+  }
+  if (lane == 0) {
+    sh.red_m[warp] = m;
+    sh.red_z[warp] = z;
+    sh.red_i[warp] = mi;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    float M = sh.red_m[0], Z = sh.red_z[0];
+    int32_t A = sh.red_i[0];
+    for (int w = 1; w < kSoftThreads / 32; ++w) {
+      const float om = sh.red_m[w], oz = sh.red_z[w];
+      const float nm = fmaxf(M, om);
+      Z = (M == -INFINITY ? 0.f : Z * expf(M - nm)) + (om == -INFINITY ? 0.f : oz * expf(om - nm));
+      if (om > M || (om == M && sh.red_i[w] < A)) A = sh.red_i[w];
+      M = nm;
+    }
+    sh.M = M;
+    sh.Z = Z;
+    sh.y = A;
+    const rgd_gate_state& s = sh.s;
+    const bool stop = eos >= 0 && A == eos;
+    const bool compatible = s.confirmed || find_child(t, s.node, A) >= 0;
+    sh.mode = (s.steps >= c || stop || compatible) ? 1 : 2;  // 1: the hard step with y; 2: the soft branch
+    if (sh.mode == 2) {
+      // the candidates: children of the node (and the stop token) inside the vocabulary
+      const int32_t b = __ldg(t.child_begin + s.node), e = __ldg(t.child_begin + s.node + 1);
+      int32_t n = 0;
+      for (int32_t k = b; k < e; ++k) {
+        const int32_t a = __ldg(t.child_tok + k);
+        if (a >= 0 && a < vocab && a != eos) sh.key[n++] = rank_key(logit_at<LT>(row, a), a);
+      }
+      if (eos >= 0 && eos < vocab) sh.key[n++] = rank_key(logit_at<LT>(row, eos), eos);
+      sh.ncand = n;
+    }
+  }
+  __syncthreads();
+  if (sh.mode == 2) {
+    // ---- sort the candidates (bitonic, padded to a power of two) ----
+    const int32_t n = sh.ncand;
+    int32_t np = 1;
+    while (np < n) np <<= 1;
+    for (int32_t i = n + tid; i < np; i += kSoftThreads) sh.key[i] = ~0ull;
+    __syncthreads();
+    for (int32_t k = 2; k <= np; k <<= 1) {
+      for (int32_t j = k >> 1; j > 0; j >>= 1) {
+        for (int32_t i = tid; i < np; i += kSoftThreads) {
+          const int32_t ij = i ^ j;
+          if (ij > i) {
+            const uint64_t a = sh.key[i], b2 = sh.key[ij];
+            if ((a > b2) == ((i & k) == 0)) {
+              sh.key[i] = b2;
+              sh.key[ij] = a;
+            }
+          }
+        }
+        __syncthreads();
+      }
+    }
+    // ---- ranks of the candidates, kChunk per pass, until one leaves the top K ----
+    if (tid == 0) {
+      sh.n_in = 0;
+      sh.stop = 0;
+      sh.mass = 0.f;
+    }
+    __syncthreads();
+    const int32_t limit = min(n, top_k);
+    for (int32_t c0 = 0; c0 < limit; c0 += kChunk) {
+      const int32_t nc = min(kChunk, limit - c0);
+      if (tid < kChunk) {
+        const uint64_t key = tid < nc ? sh.key[c0 + tid] : ~0ull;
+        sh.cv[tid] = tid < nc ? key_logit(key) : INFINITY;  // (padding: nothing ranks above it)
+        sh.ci[tid] = tid < nc ? (int32_t)(uint32_t)key : -1;
+        sh.cnt[tid] = 0;
+      }
+      __syncthreads();
+      int32_t cn[kChunk];
+#pragma unroll
+      for (int k = 0; k < kChunk; ++k) cn[k] = 0;
+      for (int32_t i = tid; i < vocab; i += kSoftThreads) {
+        const float v = logit_at<LT>(row, i);
+#pragma unroll
+        for (int k = 0; k < kChunk; ++k) cn[k] += above(v, i, sh.cv[k], sh.ci[k]) ? 1 : 0;
+      }
+#pragma unroll
+      for (int k = 0; k < kChunk; ++k) {
+        int32_t x = cn[k];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+        if (lane == 0 && x) atomicAdd(&sh.cnt[k], x);
+      }
+      __syncthreads();
+      if (tid == 0) {
+        for (int k = 0; k < nc && !sh.stop; ++k) {
+          if (sh.cnt[k] >= top_k) {
+            sh.stop = 1;
+          } else {
+            sh.mass += expf(sh.cv[k] - sh.M) / sh.Z;
+            ++sh.n_in;
+          }
+        }
+      }
+      __syncthreads();
+      if (sh.stop) break;
+    }
+  }
+  if (tid != 0) return;
+  // ---- the step's outcome ----
+  rgd_gate_state s = sh.s;
+  const bool root_has_children = __ldg(t.child_begin + 1) > __ldg(t.child_begin);
+  int32_t tok = -1;
+  if (sh.mode == 1) {
+    tok = sh.y;
+    consume_token(t, s, tok, eos, max_len, root_has_children);
+  } else if (sh.n_in > 0 && sh.mass >= rho) {
+    tok = (int32_t)(uint32_t)sh.key[0];  // a*: the most probable compatible token
+    consume_token(t, s, tok, eos, max_len, root_has_children);
+  } else {  // no refusal-like alternative with enough mass: discard the probe
+    s.decision = RGD_NON_REFUSAL;
+    s.decisive_step = s.steps;
+    s.steps++;
+    s.done = 1;
+  }
+  state[g] = s;
+  token_out[g] = tok;
+  if (mass_out) mass_out[g] = sh.mode == 2 ? sh.mass : -1.f;
+  mask_rows(s, row_active, g, rows_per_group);
 }
 
 }  // namespace
@@ -169,7 +415,9 @@ extern "C" int rgd_trie_create(const int32_t* tokens, const int64_t* offsets, in
   const int32_t nn = (int32_t)kids.size();
   std::vector<int32_t> begin(nn + 1, 0), ctok, cnode;
   std::vector<uint8_t> confirm(nn, 0);
+  int32_t max_children = 0;
   for (int32_t n = 0; n < nn; ++n) {
+    max_children = std::max(max_children, (int32_t)kids[n].size());
     begin[n] = (int32_t)ctok.size();
     for (const auto& kv : kids[n]) {
       ctok.push_back(kv.first);
@@ -185,6 +433,7 @@ extern "C" int rgd_trie_create(const int32_t* tokens, const int64_t* offsets, in
   rgd_trie* t = new rgd_trie();
   t->num_nodes = nn;
   t->num_edges = begin[nn];
+  t->max_children = max_children;
   cudaGetDevice(&t->device);
   cudaError_t err = cudaSuccess;
   auto upload = [&](void** dst, const void* src, size_t bytes) {
@@ -251,4 +500,39 @@ extern "C" int rgd_probe_gate(const rgd_trie* trie, int32_t groups, int32_t rows
       dev_status);
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? RGD_OK : cuda_error(e, "probe_gate launch");
+}
+
+extern "C" int rgd_soft_gate(const rgd_trie* trie, int32_t groups, int32_t rows_per_group, int32_t vocab,
+                             int32_t dtype, const void* probe_logits, int64_t row_stride, int32_t top_k, float rho,
+                             int32_t c, int32_t eos_token, int32_t max_len, rgd_gate_state* state,
+                             uint8_t* row_active, int32_t* token_out, float* mass_out, int32_t* dev_status,
+                             rgd_stream_t stream) {
+  clear_error();
+  (void)dev_status;
+  RGD_CHECK_ARG(trie != nullptr, "rgd_soft_gate: trie is NULL");
+  RGD_CHECK_ARG(groups >= 0 && rows_per_group >= 1 && vocab >= 1, "rgd_soft_gate: bad groups/rows/vocab");
+  RGD_CHECK_ARG(dtype == RGD_F32 || dtype == RGD_BF16, "rgd_soft_gate: dtype must be RGD_F32 or RGD_BF16");
+  RGD_CHECK_ARG(row_stride >= vocab, "rgd_soft_gate: row_stride < vocab");
+  RGD_CHECK_ARG(top_k >= 1 && c >= 0 && max_len >= 1, "rgd_soft_gate: need top_k >= 1, c >= 0, max_len >= 1");
+  RGD_CHECK_ARG(std::isfinite(rho), "rgd_soft_gate: rho must be finite");
+  if (trie->max_children + 1 > kMaxCand)
+    return set_error(RGD_ERR_UNSUPPORTED, "rgd_soft_gate: a trie node has %d children (max %d)",
+                     trie->max_children, kMaxCand - 1);
+  if (groups == 0) return RGD_OK;
+  RGD_CHECK_ARG(probe_logits != nullptr && state != nullptr && token_out != nullptr,
+                "rgd_soft_gate: logits/state/token_out NULL");
+  TrieView tv{trie->child_begin, trie->child_tok, trie->child_node, trie->confirm};
+  cudaStream_t st = (cudaStream_t)stream;
+  if (dtype == RGD_F32)
+    soft_gate_kernel<float><<<groups, kSoftThreads, 0, st>>>(tv, rows_per_group, vocab,
+                                                              static_cast<const float*>(probe_logits), row_stride,
+                                                              top_k, rho, c, eos_token, max_len, state, row_active,
+                                                              token_out, mass_out);
+  else
+    soft_gate_kernel<uint16_t><<<groups, kSoftThreads, 0, st>>>(tv, rows_per_group, vocab,
+                                                                 static_cast<const uint16_t*>(probe_logits),
+                                                                 row_stride, top_k, rho, c, eos_token, max_len,
+                                                                 state, row_active, token_out, mass_out);
+  cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? RGD_OK : cuda_error(e, "soft_gate launch");
 }

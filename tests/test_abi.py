@@ -53,6 +53,12 @@ def test_version_and_argument_errors_without_gpu(lib_path):
     rc = lib.rgd_residual_precheck(4, 16, 0, None, None, 0.0, 0.5, 5, None, None, None, None, None)
     assert rc == binding.RGD_ERR_INVALID_ARG
     assert lib.rgd_residual_precheck(0, 16, 0, None, None, 0.0, 0.5, 5, None, None, None, None, None) == 0
+    # the soft gate: a NULL trie, top_k < 1
+    rc = lib.rgd_soft_gate(None, 1, 1, 10, 0, None, 10, 5, 0.1, 2, -1, 8, None, None, None, None, None, None)
+    assert rc == binding.RGD_ERR_INVALID_ARG
+    # (the argument checks come before the trie is looked at: any non-NULL handle does here)
+    rc = lib.rgd_soft_gate(1, 1, 1, 10, 0, 1, 10, 0, 0.1, 2, -1, 8, 1, None, 1, None, None, None)
+    assert rc == binding.RGD_ERR_INVALID_ARG and b"top_k" in lib.rgd_last_error_string()
 
 
 def test_workspace_size_grows_with_blocks(lib_path):
