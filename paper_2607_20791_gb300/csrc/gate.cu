@@ -153,24 +153,20 @@ __global__ void probe_gate_kernel(TrieView t, int32_t groups, int32_t rows_per_g
 // One block per group.  Pass 1 reads the probe's logits once: the maximum, its
 // lowest index (y) and the softmax normaliser Z (per-thread online sums).  The
 // soft branch then sorts the compatible candidates by logit in shared memory
-// (bitonic sort of (logit, token) keys) and counts, in passes over the logits
-// (from L2), how many tokens rank above each of the next 32 candidates; the
-// ranks grow along the sorted order, so the counting stops at the first
-// candidate outside the top K.
+// (bitonic sort of (logit, token) keys); their ranks grow along that order,
+// so a binary search over it, one pass over the logits (from L2) per probed
+// candidate, finds how many of them are in the top K.
 constexpr int kSoftThreads = 512;
 constexpr int kMaxCand = 2048;  // a node's children + the stop token, sorted in shared memory
-constexpr int kChunk = 32;      // candidates ranked per pass over the logits
 
 struct SoftShared {
   uint64_t key[kMaxCand];
   float red_m[kSoftThreads / 32], red_z[kSoftThreads / 32];
   int32_t red_i[kSoftThreads / 32];
-  int32_t cnt[kChunk];
-  float cv[kChunk];   // the chunk's candidates: logits and tokens
-  int32_t ci[kChunk];
+  int32_t cnt[1];
   rgd_gate_state s;
   float M, Z, mass;
-  int32_t y, mode, ncand, n_in, stop;
+  int32_t y, mode, ncand, n_in;
 };
 
 template <typename LT>
@@ -182,6 +178,60 @@ __device__ __forceinline__ float logit_at<float>(const float* row, int64_t i) {
 template <>
 __device__ __forceinline__ float logit_at<uint16_t>(const uint16_t* row, int64_t i) {
   return __uint_as_float((uint32_t)__ldg(row + i) << 16);
+}
+
+// Element e of a 16-byte vector of logits.
+template <typename LT>
+__device__ __forceinline__ float vec_elem(const uint4& w, int e);
+template <>
+__device__ __forceinline__ float vec_elem<float>(const uint4& w, int e) {
+  return __uint_as_float(e == 0 ? w.x : e == 1 ? w.y : e == 2 ? w.z : w.w);
+}
+template <>
+__device__ __forceinline__ float vec_elem<uint16_t>(const uint4& w, int e) {
+  const uint32_t u = (e >> 1) == 0 ? w.x : (e >> 1) == 1 ? w.y : (e >> 1) == 2 ? w.z : w.w;
+  return __uint_as_float((e & 1) ? (u & 0xffff0000u) : (u << 16));
+}
+
+// Calls f(logit, index) for this thread's share of a row, in increasing index
+// order, with kBatchLoads loads in flight: 16-byte vectors when the row is
+// 16-byte aligned (then the few elements past the last whole vector, one per
+// thread, come last), else single elements.
+template <int kThreads, int kBatchLoads, typename LT, typename F>
+__device__ __forceinline__ void scan_row(const LT* row, int32_t vocab, bool vec, F&& f) {
+  constexpr int E = 16 / (int)sizeof(LT);
+  const int tid = threadIdx.x;
+  if (vec) {
+    const int32_t nvec = vocab / E;
+    const uint4* rv = reinterpret_cast<const uint4*>(row);
+    for (int32_t v0 = tid; v0 < nvec; v0 += kBatchLoads * kThreads) {
+      uint4 w[kBatchLoads];
+#pragma unroll
+      for (int b = 0; b < kBatchLoads; ++b)
+        if (v0 + b * kThreads < nvec) w[b] = __ldg(rv + v0 + b * kThreads);
+#pragma unroll
+      for (int b = 0; b < kBatchLoads; ++b) {
+        const int32_t vi = v0 + b * kThreads;
+        if (vi >= nvec) break;
+#pragma unroll
+        for (int e = 0; e < E; ++e) f(vec_elem<LT>(w[b], e), vi * E + e);
+      }
+    }
+    const int32_t i = nvec * E + tid;
+    if (i < vocab) f(logit_at<LT>(row, i), i);
+  } else {
+    for (int32_t i0 = tid; i0 < vocab; i0 += kBatchLoads * kThreads) {
+      float v[kBatchLoads];
+#pragma unroll
+      for (int b = 0; b < kBatchLoads; ++b)
+        if (i0 + b * kThreads < vocab) v[b] = logit_at<LT>(row, i0 + b * kThreads);
+#pragma unroll
+      for (int b = 0; b < kBatchLoads; ++b) {
+        if (i0 + b * kThreads >= vocab) break;
+        f(v[b], i0 + b * kThreads);
+      }
+    }
+  }
 }
 
 // Order-preserving key: ascending keys = logits descending, then tokens ascending.
@@ -202,7 +252,7 @@ __device__ __forceinline__ bool above(float v, int64_t i, float w, int64_t j) { 
 template <typename LT>
 __global__ void __launch_bounds__(kSoftThreads)
     soft_gate_kernel(TrieView t, int32_t rows_per_group, int32_t vocab, const LT* __restrict__ logits,
-                     int64_t row_stride, int32_t top_k, float rho, int32_t c, int32_t eos, int32_t max_len,
+                     int64_t row_stride, bool vec, int32_t top_k, float rho, int32_t c, int32_t eos, int32_t max_len,
                      rgd_gate_state* __restrict__ state, uint8_t* __restrict__ row_active, int32_t* token_out,
                      float* mass_out) {
   __shared__ SoftShared sh;
@@ -224,9 +274,7 @@ __global__ void __launch_bounds__(kSoftThreads)
   // ---- pass 1: maximum, its lowest index, and Z = sum exp(l - max) ----
   float m = -INFINITY, z = 0.f;
   int32_t mi = 0x7fffffff;
-#pragma unroll 8
-  for (int32_t i = tid; i < vocab; i += kSoftThreads) {
-    const float v = logit_at<LT>(row, i);
+  scan_row<kSoftThreads, 8, LT>(row, vocab, vec, [&](float v, int32_t i) {
     if (v > m) {  // indices grow along a thread: strict > keeps the lowest
       z = (m == -INFINITY) ? 1.f : z * expf(m - v) + 1.f;
       m = v;
@@ -234,7 +282,7 @@ __global__ void __launch_bounds__(kSoftThreads)
     } else if (m != -INFINITY) {  // (with m = -inf, v is -inf too and adds nothing)
       z += expf(v - m);
     }
-  }
+  });
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     const float om = __shfl_xor_sync(0xffffffffu, m, o), oz = __shfl_xor_sync(0xffffffffu, z, o);
@@ -302,52 +350,34 @@ __global__ void __launch_bounds__(kSoftThreads)
         __syncthreads();
       }
     }
-    // ---- ranks of the candidates, kChunk per pass, until one leaves the top K ----
+    // ---- how many of the sorted candidates are in the top K: their ranks
+    // grow along the order, so a binary search, one candidate per pass (each
+    // pass one comparison per logit, the logits read from L2) ----
+    int32_t lo = 0, hi = min(n, top_k);
+    while (lo < hi) {  // (lo, hi are the same in every thread)
+      const int32_t mid = (lo + hi) >> 1;
+      const uint64_t key = sh.key[mid];
+      const float cv = key_logit(key);
+      const int32_t ci = (int32_t)(uint32_t)key;
+      if (tid == 0) sh.cnt[0] = 0;
+      __syncthreads();
+      int32_t cnt = 0;
+      scan_row<kSoftThreads, 8, LT>(row, vocab, vec, [&](float v, int32_t i) { cnt += above(v, i, cv, ci) ? 1 : 0; });
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+      if (lane == 0 && cnt) atomicAdd(&sh.cnt[0], cnt);
+      __syncthreads();
+      if (sh.cnt[0] < top_k) lo = mid + 1;
+      else hi = mid;
+      __syncthreads();  // (sh.cnt is reset in the next pass)
+    }
     if (tid == 0) {
-      sh.n_in = 0;
-      sh.stop = 0;
-      sh.mass = 0.f;
+      sh.n_in = lo;
+      float mass = 0.f;
+      for (int k = 0; k < lo; ++k) mass += expf(key_logit(sh.key[k]) - sh.M) / sh.Z;
+      sh.mass = mass;
     }
     __syncthreads();
-    const int32_t limit = min(n, top_k);
-    for (int32_t c0 = 0; c0 < limit; c0 += kChunk) {
-      const int32_t nc = min(kChunk, limit - c0);
-      if (tid < kChunk) {
-        const uint64_t key = tid < nc ? sh.key[c0 + tid] : ~0ull;
-        sh.cv[tid] = tid < nc ? key_logit(key) : INFINITY;  // (padding: nothing ranks above it)
-        sh.ci[tid] = tid < nc ? (int32_t)(uint32_t)key : -1;
-        sh.cnt[tid] = 0;
-      }
-      __syncthreads();
-      int32_t cn[kChunk];
-#pragma unroll
-      for (int k = 0; k < kChunk; ++k) cn[k] = 0;
-      for (int32_t i = tid; i < vocab; i += kSoftThreads) {
-        const float v = logit_at<LT>(row, i);
-#pragma unroll
-        for (int k = 0; k < kChunk; ++k) cn[k] += above(v, i, sh.cv[k], sh.ci[k]) ? 1 : 0;
-      }
-#pragma unroll
-      for (int k = 0; k < kChunk; ++k) {
-        int32_t x = cn[k];
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-        if (lane == 0 && x) atomicAdd(&sh.cnt[k], x);
-      }
-      __syncthreads();
-      if (tid == 0) {
-        for (int k = 0; k < nc && !sh.stop; ++k) {
-          if (sh.cnt[k] >= top_k) {
-            sh.stop = 1;
-          } else {
-            sh.mass += expf(sh.cv[k] - sh.M) / sh.Z;
-            ++sh.n_in;
-          }
-        }
-      }
-      __syncthreads();
-      if (sh.stop) break;
-    }
   }
   if (tid != 0) return;
   // ---- the step's outcome ----
@@ -523,15 +553,17 @@ extern "C" int rgd_soft_gate(const rgd_trie* trie, int32_t groups, int32_t rows_
                 "rgd_soft_gate: logits/state/token_out NULL");
   TrieView tv{trie->child_begin, trie->child_tok, trie->child_node, trie->confirm};
   cudaStream_t st = (cudaStream_t)stream;
+  const int es = dtype == RGD_F32 ? 4 : 2;
+  const bool vec = aligned16(probe_logits) && (row_stride * es) % 16 == 0;  // 16-byte vector loads
   if (dtype == RGD_F32)
     soft_gate_kernel<float><<<groups, kSoftThreads, 0, st>>>(tv, rows_per_group, vocab,
                                                               static_cast<const float*>(probe_logits), row_stride,
-                                                              top_k, rho, c, eos_token, max_len, state, row_active,
+                                                              vec, top_k, rho, c, eos_token, max_len, state, row_active,
                                                               token_out, mass_out);
   else
     soft_gate_kernel<uint16_t><<<groups, kSoftThreads, 0, st>>>(tv, rows_per_group, vocab,
                                                                  static_cast<const uint16_t*>(probe_logits),
-                                                                 row_stride, top_k, rho, c, eos_token, max_len,
+                                                                 row_stride, vec, top_k, rho, c, eos_token, max_len,
                                                                  state, row_active, token_out, mass_out);
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? RGD_OK : cuda_error(e, "soft_gate launch");
