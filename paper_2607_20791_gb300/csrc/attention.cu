@@ -12,41 +12,46 @@
 //
 // Work distribution.  The jobs' page lists are laid end to end (job-major) and
 // the grid's persistent blocks (one per SM) each take an equal contiguous range
-// of pages.  A job split across blocks leaves a partial (o, m, l) in workspace
-// slot (block + job) -- distinct for every piece, since block ranges are ordered
-// like the jobs -- and takes a ticket; the block holding the job's last piece
-// to finish merges the partials by log-sum-exp (Sec. 3's shared-prefix split is
-// the same identity).  Only the two jobs at the ends of a block's range can be
-// split, and a block works on those two first, so the merges happen early and
-// overlap the rest of the block's work.
+// of pages.  Only the two jobs at the ends of a block's range can be split with
+// a neighbour, and a block works on those two first (the end of the job it
+// starts in, then the start of the job it ends in, then the whole jobs between).
+// A split job is merged by log-sum-exp (Sec. 3's shared-prefix split is the same
+// identity) in the block holding its first page: the job's other pieces --
+// each the first piece of its own block -- write a partial (o, m, l) to
+// workspace slot (block + job) and count themselves in the job's ticket; the
+// merger's watcher warp polls the ticket while its own piece runs, brings the
+// partials into shared memory by bulk copies once all have counted, and folds
+// them into its own O on the way out.
 //
-// Inside a block (608 threads) the tensor memory holds Q, S / P and O, so the
-// tensor cores read only K and V from shared memory -- the bytes that come from
-// HBM:
-//   * warp 16 (producer) streams the pages, four to a group, into a ring of
-//     group slots with 3-D TMA boxes (128-byte swizzle): each K tile lands as
-//     two 2 KiB halves in a half-major, group-contiguous block, so that one MMA
-//     covers all the group's tokens (an MMA costs ~50 cycles to issue whatever
-//     its N, so the number of MMAs, not their size, is what counts), each V
-//     tile as one box; every lane issues its own page, since one issuing
-//     thread is copy-rate bound;
-//   * warp 17 allocates the tensor memory and its lane 0 issues, for a group
+// Inside a block (384 threads for R = 4 query copies, 512 for 2, 640 for 1) the
+// tensor memory holds Q, S, P and O, so the tensor cores read only K and V from
+// shared memory -- the bytes that come from HBM:
+//   * two producer warps take alternate rounds of 32 pages and stream them,
+//     four to a group, into a ring of group slots with 3-D TMA boxes (128-byte
+//     swizzle): each K tile lands as two 2 KiB halves in a half-major,
+//     group-contiguous block, so that one MMA covers all the group's tokens (an
+//     MMA costs ~50 cycles to issue whatever its N, so the number of MMAs, not
+//     their size, is what counts), each V tile as one box; every lane issues
+//     its own page, since one issuing thread is copy-rate bound;
+//   * the QK warp allocates the tensor memory and its lane 0 issues, per group
 //     of up to 4 pages, S = Q K^T (A = Q from TMEM, M = 128 query rows,
-//     N = 16 x pages) into one of three S/P buffers; once the softmax warps
-//     have turned S into bf16 P in place, lane 0 of warp 18 issues O += P V per
-//     page (A = P from TMEM, N = the head dimension, V read MN-major from its
-//     tile), and one commit after the group's PV hands its slot back to the
-//     producer;
-//   * warps 0-15 (softmax): warp w can reach TMEM lanes 32(w%4)..+31 only.  The
-//     job's queries are held in as many copies as fit in the 128 lanes; a
-//     softmax warp handles the 16 scores of one page for 32 query rows of one
-//     copy: the masks, the row max (shared through shared memory by the warps of
-//     a copy that share rows), the online softmax in fp32 (the running max is
-//     only moved, and O rescaled in TMEM, when a row's max grows by more than
-//     2^8) and its 16 bf16 P values.  They also write Q into TMEM, and at the end
-//     of a job piece every warp of a used lane quarter reads a quarter of O's
-//     columns; the copies are merged by log-sum-exp and the output or the
-//     partial written.
+//     N = 16 x pages) into the S buffer; the softmax warps turn S into P (a
+//     bf16 high part and a bf16 residual, in two P buffers), and lane 0 of the
+//     PV warp issues O += P V for both parts per page (A = P from TMEM, N = the
+//     head dimension, V read MN-major from its tile); one commit after the
+//     group's PV hands its slot back to the producers;
+//   * softmax warps: warp w can reach TMEM lanes 32(w%4)..+31 only.  The job's
+//     queries are held in R copies in the 128 lanes; a softmax warp handles the
+//     16 scores of one page for 32 query rows of one copy: the masks, the row
+//     max (shared through shared memory by the warps of a copy that share
+//     rows), the online softmax in fp32 (the running max is only moved, and O
+//     rescaled in TMEM, when a row's max grows by more than 2^8) and its P;
+//   * epilogue warps (one per used lane quarter when R > 1; the softmax warps
+//     themselves when R = 1) write the next piece's Q into TMEM once the
+//     current piece's last QK is done, and at a piece's end read O (double-
+//     buffered by piece, so the softmax warps go on meanwhile), merge the copies
+//     by log-sum-exp through shared memory and write the output, the partial
+//     of a split job, or -- in a merger -- the merged output.
 // Every wait on an mbarrier is bounded; a timeout is reported in the status
 // word and every role stops.
 #include <cudaTypedefs.h>
