@@ -165,6 +165,22 @@ def _dist_env():
     return world, rank, local
 
 
+def aggregate_over_ranks(step_ms: float, e2e_ms: float, attn_ms: float, rows_per_step: int, world: int,
+                         device="cpu"):
+    """Max of the per-rank times over the job (every rank gets the same
+    result), and the whole-job throughputs: world * rows / max step time.
+    Needs an initialised process group when world > 1 (NCCL on the GPUs, gloo
+    in the CPU tests)."""
+    import torch
+    vals = torch.tensor([step_ms, e2e_ms, attn_ms], dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(vals, op=dist.ReduceOp.MAX)
+    step_ms, e2e_ms, attn_ms = [float(x) for x in vals.tolist()]
+    return {"step_ms": step_ms, "e2e_ms": e2e_ms, "attn_ms": attn_ms,
+            "value": world * rows_per_step / (step_ms / 1e3), "e2e_value": world * rows_per_step / (e2e_ms / 1e3)}
+
+
 # ---------------------------------------------------------------------------
 # CPU oracle timing (cpu_baseline leg and --impl reference)
 # ---------------------------------------------------------------------------
@@ -413,12 +429,9 @@ def run_ours(args):
     e2e_ms = sum(a.elapsed_time(b) for a, b in e2e_ev) / args.steps
 
     # ---- max over ranks --------------------------------------------------------
-    vals = torch.tensor([mean_step, e2e_ms, mean_attn], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(vals, op=dist.ReduceOp.MAX)
-    mean_step, e2e_ms, mean_attn = [float(x) for x in vals.tolist()]
-    value = world * rows_per_step / (mean_step / 1e3)
-    e2e_value = world * rows_per_step / (e2e_ms / 1e3)
+    agg = aggregate_over_ranks(mean_step, e2e_ms, mean_attn, rows_per_step, world, device=dev)
+    mean_step, e2e_ms, mean_attn = agg["step_ms"], agg["e2e_ms"], agg["attn_ms"]
+    value, e2e_value = agg["value"], agg["e2e_value"]
 
     if rank == 0:
         peak, peak_kind = _peaks()
