@@ -428,6 +428,24 @@ def run_ours(args):
         torch.cuda.synchronize()
     e2e_ms = sum(a.elapsed_time(b) for a, b in e2e_ev) / args.steps
 
+    # ---- size-matched copy (context for the roofline fraction) ------------------
+    # a plain device copy moving the attention's algorithmic byte count (half read,
+    # half written), L2 flushed before each, timed with events like the kernels:
+    # the bandwidth a transfer of this size reaches at all
+    half = (attn_bytes // 2 + 15) // 16 * 16
+    c_src = torch.ones(half, dtype=torch.uint8, device=dev)
+    c_dst = torch.empty_like(c_src)
+    c_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(12)]
+    with torch.cuda.stream(stream):
+        for a, b in c_ev:
+            flush.fill_(1)
+            a.record(stream)
+            c_dst.copy_(c_src)
+            b.record(stream)
+    torch.cuda.synchronize()
+    copy_ms = sorted(a.elapsed_time(b) for a, b in c_ev[3:])[4]
+    del c_src, c_dst
+
     # ---- max over ranks --------------------------------------------------------
     agg = aggregate_over_ranks(mean_step, e2e_ms, mean_attn, rows_per_step, world, device=dev)
     mean_step, e2e_ms, mean_attn = agg["step_ms"], agg["e2e_ms"], agg["attn_ms"]
@@ -467,6 +485,11 @@ def run_ours(args):
             "residual_precheck": {"us": 1e3 * sorted(pre_ms)[len(pre_ms) // 2], "groups": pre.groups, "d": pre.d,
                                   "bytes": pre_bytes, "bound": "launch latency (a d + 1 logistic readout)",
                                   "note": "once per prompt, outside the step"},
+            "copy_ceiling": {"bytes": 2 * half, "us": copy_ms * 1e3, "gbs": 2 * half / (copy_ms / 1e3) / 1e9,
+                             "frac_of_peak": 2 * half / (copy_ms / 1e3) / 1e9 / peak,
+                             "attention_frac_of_copy": copy_ms / mean_attn,
+                             "note": "a plain device copy of the attention's algorithmic byte count (half read, "
+                                     "half written), L2 flushed, median of 9: what a transfer of this size reaches"},
             "clocks": clocks, "dev_status": status,
         }
         print(json.dumps(line), flush=True)
