@@ -6,9 +6,9 @@
  * to the prompt's KV cache, which is computed once and reused (Sec. 3), plus
  * their own generated-suffix KV.  The greedy probe is checked token by token
  * against a set P of refusal prefixes (the compatibility predicate C, Sec. 3;
- * token-prefix matching with a two-token minimum, App. D); the hard gate of
- * Alg. 1 then either keeps the greedy refusal or discards the probe and keeps
- * the high-temperature samples.
+ * matched on token prefixes, a detection needing at least two tokens, App. D);
+ * the hard gate of Alg. 1 then either keeps the greedy refusal or discards the
+ * probe and keeps the high-temperature samples.
  *
  * This library implements one decode step of that loop as CUDA kernels:
  *   rgd_prefix_decode_attn  shared-prefix split-KV decode attention,

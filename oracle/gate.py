@@ -1,7 +1,7 @@
 """Refusal-prefix compatibility gate, oracle side (test infrastructure only).
 
-Compatibility predicate (Sec. 3): C(d(q), P) is true when d(q) is a prefix of
-some pi in P or some pi in P is already a prefix of d(q).  It is evaluated here
+Compatibility predicate (Sec. 3): C(d(q), P) holds iff d(q) begins some pi in
+P, or d(q) itself begins with some pi in P.  It is evaluated here
 on token sequences (the runtime detector's token-prefix matching, App. D), with
 the two-token minimum of App. D read as: a detection "pi is a prefix of q"
 counts only for |pi| >= min_confirm (= 2).  So

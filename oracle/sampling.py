@@ -4,8 +4,8 @@ Follows the paper's decode primitives (Sec. 3, Alg. 1):
 
 * G_M(p, q): one greedy decode step -> the argmax of the next-token logits.
   Ties are broken toward the lowest token index.
-* S_{T,theta}(M, p): ordinary high-temperature sampling at temperature T with
-  truncation parameters theta.  The truncation used here is min-p (cited in
+* S_{T,theta}(M, p): plain sampling at a high temperature T, truncated as the
+  parameters theta say.  The truncation used here is min-p (cited in
   Sec. 1 and Sec. 2): keep the tokens whose probability under softmax(l / T) is
   at least p_min times the largest probability, renormalise, draw one token.
 
