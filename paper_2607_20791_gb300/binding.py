@@ -96,7 +96,28 @@ def _check(rc: int) -> None:
         raise RgdError(rc, load_library().rgd_last_error_string().decode())
 
 
-def _ptr(t, name: str, dtype=None, optional: bool = False) -> Optional[int]:
+class _HostTensor:
+    """Stands in for the pointer of a tensor that is not on the GPU; :func:`_call`
+    refuses the call once every other argument has been checked."""
+
+    def __init__(self, name: str):
+        self.name = name
+
+
+def _call(fn, *args):
+    """Call a C entry point unless an argument is a host tensor."""
+    for a in args:
+        if isinstance(a, _HostTensor):
+            raise ValueError(f"{a.name} must be a CUDA tensor")
+    return fn(*args)
+
+
+def _ptr(t, name: str, dtype=None, optional: bool = False, numel: Optional[int] = None):
+    """Device pointer of a contiguous CUDA tensor (or a raw int pointer, passed
+    through unchecked).  ``numel`` is the number of elements the call will
+    touch: a smaller tensor is refused here, since the C side sees only the
+    pointer.  A host tensor gives a :class:`_HostTensor`, refused by
+    :func:`_call`, so that every argument's type and size is checked first."""
     if t is None:
         if optional:
             return None
@@ -106,19 +127,24 @@ def _ptr(t, name: str, dtype=None, optional: bool = False) -> Optional[int]:
     import torch
     if not isinstance(t, torch.Tensor):
         raise TypeError(f"{name}: expected a torch tensor or an int pointer")
-    if not t.is_cuda:
-        raise ValueError(f"{name} must be a CUDA tensor")
-    if not t.is_contiguous():
-        raise ValueError(f"{name} must be contiguous")
     if dtype is not None and t.dtype not in (dtype if isinstance(dtype, tuple) else (dtype,)):
         raise TypeError(f"{name}: dtype {t.dtype} not accepted")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if numel is not None and t.numel() < numel:
+        raise ValueError(f"{name} holds {t.numel()} elements, the call needs {numel}")
+    if not t.is_cuda:
+        return _HostTensor(name)
     return t.data_ptr()
 
 
 def _stream(stream) -> Optional[int]:
     if stream is None:
         import torch
-        return torch.cuda.current_stream().cuda_stream
+        try:
+            return torch.cuda.current_stream().cuda_stream
+        except (RuntimeError, AssertionError):  # no CUDA device: the call is refused or fails in CUDA
+            return None
     if isinstance(stream, int):
         return stream
     return stream.cuda_stream
@@ -135,20 +161,32 @@ def rgd_prefix_decode_attn_workspace_size(shape: AttnShape) -> int:
     return int(n)
 
 
+def _attn_sizes(shape: AttnShape) -> dict:
+    """Elements each attention argument must hold for ``shape``."""
+    R = shape.num_groups * shape.rows_per_group
+    return {"q": R * shape.num_q_heads * shape.head_dim,
+            "kv": shape.num_pages * shape.num_kv_heads * shape.page_size * shape.head_dim,
+            "pbt": shape.num_groups * shape.max_prompt_pages, "plen": shape.num_groups,
+            "sbt": R * shape.max_suffix_pages, "rows": R, "lse": R * shape.num_q_heads}
+
+
 def rgd_prefix_decode_attn(shape: AttnShape, q, k_pages, v_pages, prompt_block_table, prompt_len,
                            suffix_block_table, suffix_len, row_active, softmax_scale: float, out, lse,
                            workspace, dev_status=None, stream=None) -> None:
     import torch
     lib = load_library()
+    n = _attn_sizes(shape)
     ws_bytes = workspace.numel() * workspace.element_size() if isinstance(workspace, torch.Tensor) else 0
-    _check(lib.rgd_prefix_decode_attn(
-        ctypes.byref(shape), _ptr(q, "q", torch.bfloat16), _ptr(k_pages, "k_pages", torch.bfloat16),
-        _ptr(v_pages, "v_pages", torch.bfloat16), _ptr(prompt_block_table, "prompt_block_table", torch.int32),
-        _ptr(prompt_len, "prompt_len", torch.int32),
-        _ptr(suffix_block_table, "suffix_block_table", torch.int32), _ptr(suffix_len, "suffix_len", torch.int32),
-        _ptr(row_active, "row_active", torch.uint8, optional=True), float(softmax_scale),
-        _ptr(out, "out", torch.bfloat16), _ptr(lse, "lse", torch.float32, optional=True),
-        _ptr(workspace, "workspace"), ws_bytes, _ptr(dev_status, "dev_status", torch.int32, optional=True),
+    _check(_call(lib.rgd_prefix_decode_attn,
+        ctypes.byref(shape), _ptr(q, "q", torch.bfloat16, numel=n["q"]),
+        _ptr(k_pages, "k_pages", torch.bfloat16, numel=n["kv"]), _ptr(v_pages, "v_pages", torch.bfloat16, numel=n["kv"]),
+        _ptr(prompt_block_table, "prompt_block_table", torch.int32, numel=n["pbt"]),
+        _ptr(prompt_len, "prompt_len", torch.int32, numel=n["plen"]),
+        _ptr(suffix_block_table, "suffix_block_table", torch.int32, numel=n["sbt"]),
+        _ptr(suffix_len, "suffix_len", torch.int32, numel=n["rows"]),
+        _ptr(row_active, "row_active", torch.uint8, optional=True, numel=n["rows"]), float(softmax_scale),
+        _ptr(out, "out", torch.bfloat16, numel=n["q"]), _ptr(lse, "lse", torch.float32, optional=True, numel=n["lse"]),
+        _ptr(workspace, "workspace"), ws_bytes, _ptr(dev_status, "dev_status", torch.int32, optional=True, numel=1),
         _stream(stream)))
 
 
@@ -158,14 +196,17 @@ def rgd_prefix_decode_attn_noalloc(shape: AttnShape, q, k_pages, v_pages, prompt
     """Same as :func:`rgd_prefix_decode_attn` without a workspace: the library's
     fixed device scratch is used (for callers that cannot allocate device memory)."""
     import torch
-    _check(load_library().rgd_prefix_decode_attn_noalloc(
-        ctypes.byref(shape), _ptr(q, "q", torch.bfloat16), _ptr(k_pages, "k_pages", torch.bfloat16),
-        _ptr(v_pages, "v_pages", torch.bfloat16), _ptr(prompt_block_table, "prompt_block_table", torch.int32),
-        _ptr(prompt_len, "prompt_len", torch.int32),
-        _ptr(suffix_block_table, "suffix_block_table", torch.int32), _ptr(suffix_len, "suffix_len", torch.int32),
-        _ptr(row_active, "row_active", torch.uint8, optional=True), float(softmax_scale),
-        _ptr(out, "out", torch.bfloat16), _ptr(lse, "lse", torch.float32, optional=True),
-        _ptr(dev_status, "dev_status", torch.int32, optional=True), _stream(stream)))
+    n = _attn_sizes(shape)
+    _check(_call(load_library().rgd_prefix_decode_attn_noalloc,
+        ctypes.byref(shape), _ptr(q, "q", torch.bfloat16, numel=n["q"]),
+        _ptr(k_pages, "k_pages", torch.bfloat16, numel=n["kv"]), _ptr(v_pages, "v_pages", torch.bfloat16, numel=n["kv"]),
+        _ptr(prompt_block_table, "prompt_block_table", torch.int32, numel=n["pbt"]),
+        _ptr(prompt_len, "prompt_len", torch.int32, numel=n["plen"]),
+        _ptr(suffix_block_table, "suffix_block_table", torch.int32, numel=n["sbt"]),
+        _ptr(suffix_len, "suffix_len", torch.int32, numel=n["rows"]),
+        _ptr(row_active, "row_active", torch.uint8, optional=True, numel=n["rows"]), float(softmax_scale),
+        _ptr(out, "out", torch.bfloat16, numel=n["q"]), _ptr(lse, "lse", torch.float32, optional=True, numel=n["lse"]),
+        _ptr(dev_status, "dev_status", torch.int32, optional=True, numel=1), _stream(stream)))
 
 
 def rgd_sample_head(logits, is_probe, temperature, min_p, seed, step: int, row_active, token_out,
@@ -177,14 +218,16 @@ def rgd_sample_head(logits, is_probe, temperature, min_p, seed, step: int, row_a
     if dtype is None:
         raise TypeError("logits must be float32 or bfloat16")
     rows, vocab = logits.shape
-    _check(load_library().rgd_sample_head(
-        rows, vocab, dtype, _ptr(logits, "logits"), _ptr(is_probe, "is_probe", torch.uint8, optional=True),
-        _ptr(temperature, "temperature", torch.float32), _ptr(min_p, "min_p", torch.float32),
-        _ptr(seed, "seed", (torch.int64, torch.uint64)), int(step) & 0xFFFFFFFFFFFFFFFF,
-        _ptr(row_active, "row_active", torch.uint8, optional=True), _ptr(token_out, "token_out", torch.int32),
-        _ptr(kept_count, "kept_count", torch.int32, optional=True),
-        _ptr(kept_mask, "kept_mask", torch.uint8, optional=True),
-        _ptr(dev_status, "dev_status", torch.int32, optional=True), _stream(stream)))
+    _check(_call(load_library().rgd_sample_head,
+        rows, vocab, dtype, _ptr(logits, "logits"),
+        _ptr(is_probe, "is_probe", torch.uint8, optional=True, numel=rows),
+        _ptr(temperature, "temperature", torch.float32, numel=rows), _ptr(min_p, "min_p", torch.float32, numel=rows),
+        _ptr(seed, "seed", (torch.int64, torch.uint64), numel=rows), int(step) & 0xFFFFFFFFFFFFFFFF,
+        _ptr(row_active, "row_active", torch.uint8, optional=True, numel=rows),
+        _ptr(token_out, "token_out", torch.int32, numel=rows),
+        _ptr(kept_count, "kept_count", torch.int32, optional=True, numel=rows),
+        _ptr(kept_mask, "kept_mask", torch.uint8, optional=True, numel=rows * vocab),
+        _ptr(dev_status, "dev_status", torch.int32, optional=True, numel=1), _stream(stream)))
 
 
 class Trie:
@@ -226,19 +269,27 @@ def rgd_trie_create(sequences, min_confirm: int = 2) -> Trie:
     return Trie(sequences, min_confirm)
 
 
+def _state_ptr(state, groups: int) -> Optional[int]:
+    """A gate-state buffer must hold ``groups`` states of GATE_STATE_BYTES each."""
+    import torch
+    return _ptr(state, "state", torch.uint8, numel=max(int(groups), 0) * GATE_STATE_BYTES)
+
+
 def rgd_gate_state_init(state, groups: int, stream=None) -> None:
-    _check(load_library().rgd_gate_state_init(_ptr(state, "state"), int(groups), _stream(stream)))
+    _check(_call(load_library().rgd_gate_state_init, _state_ptr(state, groups), int(groups), _stream(stream)))
 
 
 def rgd_probe_gate(trie: Trie, groups: int, rows_per_group: int, probe_tokens, n_tokens: int,
                    token_stride: int, eos_token: int, max_len: int, state, row_active=None,
                    dev_status=None, stream=None) -> None:
     import torch
-    _check(load_library().rgd_probe_gate(
-        trie.handle, int(groups), int(rows_per_group), _ptr(probe_tokens, "probe_tokens", torch.int32),
-        int(n_tokens), int(token_stride), int(eos_token), int(max_len), _ptr(state, "state"),
-        _ptr(row_active, "row_active", torch.uint8, optional=True),
-        _ptr(dev_status, "dev_status", torch.int32, optional=True), _stream(stream)))
+    G, rpg = int(groups), int(rows_per_group)
+    tok_n = (G - 1) * int(token_stride) + int(n_tokens) if G > 0 else 0
+    _check(_call(load_library().rgd_probe_gate,
+        trie.handle, G, rpg, _ptr(probe_tokens, "probe_tokens", torch.int32, numel=tok_n),
+        int(n_tokens), int(token_stride), int(eos_token), int(max_len), _state_ptr(state, G),
+        _ptr(row_active, "row_active", torch.uint8, optional=True, numel=G * rpg),
+        _ptr(dev_status, "dev_status", torch.int32, optional=True, numel=1), _stream(stream)))
 
 
 def rgd_residual_precheck(h, w, bias: float, theta: float, rows_per_group: int, state, row_active=None,
@@ -250,11 +301,12 @@ def rgd_residual_precheck(h, w, bias: float, theta: float, rows_per_group: int, 
     if dtype is None:
         raise TypeError("h must be float32 or bfloat16")
     groups, d = h.shape
-    _check(load_library().rgd_residual_precheck(
-        int(groups), int(d), dtype, _ptr(h, "h"), _ptr(w, "w", torch.float32), float(bias), float(theta),
-        int(rows_per_group), _ptr(prob_out, "prob_out", torch.float32, optional=True), _ptr(state, "state"),
-        _ptr(row_active, "row_active", torch.uint8, optional=True),
-        _ptr(dev_status, "dev_status", torch.int32, optional=True), _stream(stream)))
+    rpg = int(rows_per_group)
+    _check(_call(load_library().rgd_residual_precheck,
+        int(groups), int(d), dtype, _ptr(h, "h"), _ptr(w, "w", torch.float32, numel=d), float(bias), float(theta),
+        rpg, _ptr(prob_out, "prob_out", torch.float32, optional=True, numel=groups), _state_ptr(state, groups),
+        _ptr(row_active, "row_active", torch.uint8, optional=True, numel=groups * rpg),
+        _ptr(dev_status, "dev_status", torch.int32, optional=True, numel=1), _stream(stream)))
 
 
 def rgd_soft_gate(trie: Trie, groups: int, rows_per_group: int, logits, row_stride: int, top_k: int, rho: float,
@@ -267,12 +319,15 @@ def rgd_soft_gate(trie: Trie, groups: int, rows_per_group: int, logits, row_stri
     if dtype is None:
         raise TypeError("logits must be float32 or bfloat16")
     vocab = logits.shape[-1]
-    _check(load_library().rgd_soft_gate(
-        trie.handle, int(groups), int(rows_per_group), int(vocab), dtype, _ptr(logits, "logits"), int(row_stride),
-        int(top_k), float(rho), int(c), int(eos_token), int(max_len), _ptr(state, "state"),
-        _ptr(row_active, "row_active", torch.uint8, optional=True), _ptr(token_out, "token_out", torch.int32),
-        _ptr(mass_out, "mass_out", torch.float32, optional=True),
-        _ptr(dev_status, "dev_status", torch.int32, optional=True), _stream(stream)))
+    G, rpg = int(groups), int(rows_per_group)
+    log_n = (G - 1) * int(row_stride) + int(vocab) if G > 0 else 0
+    _check(_call(load_library().rgd_soft_gate,
+        trie.handle, G, rpg, int(vocab), dtype, _ptr(logits, "logits", numel=log_n), int(row_stride),
+        int(top_k), float(rho), int(c), int(eos_token), int(max_len), _state_ptr(state, G),
+        _ptr(row_active, "row_active", torch.uint8, optional=True, numel=G * rpg),
+        _ptr(token_out, "token_out", torch.int32, numel=G),
+        _ptr(mass_out, "mass_out", torch.float32, optional=True, numel=G),
+        _ptr(dev_status, "dev_status", torch.int32, optional=True, numel=1), _stream(stream)))
 
 
 def new_gate_state(groups: int, device="cuda"):

@@ -73,3 +73,69 @@ def test_workspace_size_grows_with_blocks(lib_path):
     assert grow <= b - a < grow + 512  # each region is padded to 256 bytes
     s.reserved = 1
     assert lib.rgd_prefix_decode_attn_workspace_size(ctypes.byref(s)) == 0
+
+
+def test_binding_refuses_undersized_tensors(lib_path):
+    """The C side sees only pointers, so the binding checks every tensor's size
+    against the shape before the call (CPU tensors reach that check before the
+    device check, so this runs without a GPU)."""
+    torch = pytest.importorskip("torch")
+    binding.load_library(lib_path)
+    shape = binding.AttnShape(num_groups=2, rows_per_group=3, num_q_heads=8, num_kv_heads=2, head_dim=64,
+                              page_size=16, num_pages=10, max_prompt_pages=4, max_suffix_pages=2, num_ctas=4)
+    R = 6
+    bf, i32, u8, f32 = torch.bfloat16, torch.int32, torch.uint8, torch.float32
+    good = dict(q=torch.empty(R * 8 * 64, dtype=bf), k_pages=torch.empty(10 * 2 * 16 * 64, dtype=bf),
+                v_pages=torch.empty(10 * 2 * 16 * 64, dtype=bf), prompt_block_table=torch.empty(8, dtype=i32),
+                prompt_len=torch.empty(2, dtype=i32), suffix_block_table=torch.empty(R * 2, dtype=i32),
+                suffix_len=torch.empty(R, dtype=i32), row_active=torch.empty(R, dtype=u8), softmax_scale=0.125,
+                out=torch.empty(R * 8 * 64, dtype=bf), lse=torch.empty(R * 8, dtype=f32))
+    for name in ("q", "k_pages", "prompt_block_table", "prompt_len", "suffix_block_table", "suffix_len",
+                 "row_active", "out", "lse"):
+        args = dict(good)
+        args[name] = good[name][:-1]
+        with pytest.raises(ValueError, match=name):
+            binding.rgd_prefix_decode_attn_noalloc(shape, **args)
+    # with every size right, the next check is the device one
+    with pytest.raises(ValueError, match="CUDA"):
+        binding.rgd_prefix_decode_attn_noalloc(shape, **good)
+
+    rows, vocab = 4, 50
+    head = dict(logits=torch.empty(rows, vocab), is_probe=torch.empty(rows, dtype=u8),
+                temperature=torch.empty(rows), min_p=torch.empty(rows), seed=torch.empty(rows, dtype=torch.int64),
+                step=0, row_active=torch.empty(rows, dtype=u8), token_out=torch.empty(rows, dtype=i32),
+                kept_count=torch.empty(rows, dtype=i32), kept_mask=torch.empty(rows * vocab, dtype=u8))
+    for name in ("is_probe", "temperature", "min_p", "seed", "row_active", "token_out", "kept_count", "kept_mask"):
+        args = dict(head)
+        args[name] = head[name][:-1]
+        with pytest.raises(ValueError, match=name):
+            binding.rgd_sample_head(**args)
+
+    class _NoTrie:
+        handle = None
+    st = torch.empty(3 * binding.GATE_STATE_BYTES - 1, dtype=u8)
+    with pytest.raises(ValueError, match="state"):
+        binding.rgd_gate_state_init(st, 3)
+    with pytest.raises(ValueError, match="probe_tokens"):
+        binding.rgd_probe_gate(_NoTrie(), 3, 2, torch.empty(2 * 5 + 3, dtype=i32), 4, 5, -1, 8, st)
+    with pytest.raises(ValueError, match="logits"):
+        binding.rgd_soft_gate(_NoTrie(), 3, 2, torch.empty(5 * 10 - 1), 20, 5, 0.1, 2, -1, 8, st,
+                              torch.empty(3, dtype=i32))
+    with pytest.raises(ValueError, match="w"):
+        binding.rgd_residual_precheck(torch.empty(3, 16), torch.empty(15), 0.0, 0.5, 2, st)
+
+
+def test_empty_batches_return_ok_without_a_launch(lib_path):
+    """Zero rows or groups (or no tokens this call) is a valid call that does
+    nothing; the pointers are not looked at."""
+    lib = binding.load_library(lib_path)
+    assert lib.rgd_sample_head(0, 100, 0, None, None, None, None, None, 0, None, None, None, None, None, None) == 0
+    assert lib.rgd_gate_state_init(None, 0, None) == 0
+    # (a non-NULL trie handle is required; it is not looked at for an empty call)
+    assert lib.rgd_probe_gate(1, 0, 2, None, 1, 1, -1, 8, None, None, None, None) == 0
+    assert lib.rgd_probe_gate(1, 4, 2, None, 0, 0, -1, 8, None, None, None, None) == 0
+    assert lib.rgd_residual_precheck(0, 8, 1, None, None, 0.0, 0.5, 2, None, None, None, None, None) == 0
+    # num_groups = 0 is an argument error for the attention call (its shape needs a group)
+    shape = binding.AttnShape(num_groups=0, rows_per_group=1, num_q_heads=4, num_kv_heads=1, head_dim=128,
+                              page_size=16, num_pages=1, max_prompt_pages=1, max_suffix_pages=1)
+    assert lib.rgd_prefix_decode_attn_workspace_size(ctypes.byref(shape)) == 0

@@ -53,6 +53,9 @@ def test_noalloc_rejects_oversized_shapes(gpu_lib):
     assert binding.rgd_prefix_decode_attn_workspace_size(shape) > (8 << 20)
     t = torch.zeros(16, dtype=torch.int32, device="cuda")
     b = torch.zeros(16, dtype=torch.bfloat16, device="cuda")
+    # raw pointers: the binding passes them through unchecked, so this reaches
+    # the library's own workspace check, which comes before any launch
+    tp, bp = t.data_ptr(), b.data_ptr()
     with pytest.raises(binding.RgdError) as ei:
-        binding.rgd_prefix_decode_attn_noalloc(shape, b, b, b, t, t, t, t, None, 0.1, b, None)
+        binding.rgd_prefix_decode_attn_noalloc(shape, bp, bp, bp, tp, tp, tp, tp, None, 0.1, bp, None)
     assert ei.value.code == binding.RGD_ERR_UNSUPPORTED
