@@ -3,8 +3,8 @@
 App. A replaces the greedy probe of a prompt, when a linear classifier on the
 residual stream says a refusal is unlikely: a logistic regression with d + 1
 parameters reads the d-dimensional activation h of the prompt's last token at
-one layer, and the probe is skipped (the prompt decodes directly at high
-temperature) when the predicted refusal probability is at most the calibrated
+one layer, and the probe is skipped (the prompt goes straight to
+high-temperature sampling) when the predicted refusal probability is at most the calibrated
 threshold theta.
 
     z = w . h + b,   p = sigmoid(z) = 1 / (1 + exp(-z)),   skip  <=>  p <= theta

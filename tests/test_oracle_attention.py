@@ -118,6 +118,44 @@ def test_matches_torch_sdpa_fp64():
             assert np.allclose(lse[r, h * 4:(h + 1) * 4], torch.logsumexp(s, dim=0).numpy(), atol=1e-12)
 
 
+def test_paged_layout_against_dense_tokens():
+    # the tokens are drawn first as dense [T, D] arrays in sequence order and then
+    # scattered into the page pool by this test (token t of a sequence -> page
+    # table[t // 16], slot t % 16); the oracle's gather must give attention over
+    # the dense arrays (torch fp64), across page boundaries and partial last pages
+    torch = pytest.importorskip("torch")
+    G, rpg, Hq, Hkv, D = 2, 2, 4, 2, 16
+    plens, slens = (37, 16), (0, 21, 5, 33)
+    case = workloads.make_attn_case("dense", G, rpg, Hq, Hkv, D, plens, slens, seed=11)
+    rng = np.random.default_rng(12)
+    bf = lambda shape: f32_to_bf16_bits(rng.standard_normal(shape).astype(np.float32))
+    case.k_pages[:] = 0
+    case.v_pages[:] = 0
+    dense = {}
+    for kind, table, lens in (("p", case.prompt_block_table, plens), ("s", case.suffix_block_table, slens)):
+        for i, n in enumerate(lens):
+            K, V = bf((Hkv, n, D)), bf((Hkv, n, D))
+            dense[kind, i] = (K, V)
+            for t in range(n):
+                case.k_pages[table[i, t // 16], :, t % 16] = K[:, t]
+                case.v_pages[table[i, t // 16], :, t % 16] = V[:, t]
+    o, lse = attention.decode_attention_case(case)
+    q = bf16_bits_to_f32(case.q).astype(np.float64)
+    for r in range(G * rpg):
+        Kp, Vp = dense["p", r // rpg]
+        Ks, Vs = dense["s", r]
+        for j in range(Hq):
+            h = j // (Hq // Hkv)
+            K = bf16_bits_to_f32(np.concatenate([Kp[h], Ks[h]])).astype(np.float64)
+            V = bf16_bits_to_f32(np.concatenate([Vp[h], Vs[h]])).astype(np.float64)
+            qs = torch.from_numpy(q[r, j])[None, None, None, :]
+            ref = torch.nn.functional.scaled_dot_product_attention(
+                qs, torch.from_numpy(K)[None, None], torch.from_numpy(V)[None, None], scale=case.softmax_scale)
+            assert np.allclose(o[r, j], ref[0, 0, 0].numpy(), atol=1e-12), (r, j)
+            s = case.softmax_scale * (K @ q[r, j])
+            assert lse[r, j] == pytest.approx(float(torch.logsumexp(torch.from_numpy(s), 0)), abs=1e-12)
+
+
 def test_split_merge_identity():
     # attention over [prompt | suffix] = log-sum-exp merge of attention over each part
     case = _case(G=1, rpg=3, plens=(45,), slens=(9, 0, 31))

@@ -54,6 +54,16 @@ def test_threshold_extremes():
     assert np.all(skip)  # every probability is <= 1
 
 
+def test_threshold_is_inclusive():
+    # App. A skips when the predicted probability is at most theta: at z = 0 the
+    # logistic is exactly 1/2, so theta = 1/2 skips and the next double below does not
+    h, w = np.ones((2, 8)), np.zeros(8)
+    z, p, skip = precheck.precheck(h, w, 0.0, 0.5)
+    assert np.all(z == 0.0) and np.all(p == 0.5) and np.all(skip)
+    _, _, skip = precheck.precheck(h, w, 0.0, np.nextafter(0.5, 0.0))
+    assert not np.any(skip)
+
+
 def test_apply_masks_only_skipped_fresh_groups():
     states = [ogate.GateState() for _ in range(4)]
     states[3].steps = 1  # a probe that already started is left alone

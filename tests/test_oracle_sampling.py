@@ -115,6 +115,13 @@ def test_temperature_to_zero_is_greedy():
 def test_probe_rows_ignore_temperature():
     row = np.array([0.0, 3.0, 1.0], np.float32)
     assert sampling.sample_row(row, True, 5.0, 0.0, 1, 1).token == 1
+    # 64 nearly equal logits: a T = 5 draw lands on the maximum ~1.7 % of the
+    # time, a probe row (G_M, greedy) always does
+    row = np.zeros(64, np.float32)
+    row[17] = 0.5
+    for seed in range(20):
+        assert sampling.sample_row(row, True, 5.0, 0.0, seed, 1).token == 17
+        assert sampling.sample_row(row, True, 5.0, 0.3, seed, 1).kept is None
 
 
 def test_draw_frequencies_match_weights():
