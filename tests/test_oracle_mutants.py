@@ -109,6 +109,11 @@ MUTANTS = {
     "soft_ties_to_higher_index": ("soft_gate", "test_oracle_soft_gate", "osg",
                                   [("order = np.lexsort((np.arange(l.size), -l))",
                                     "order = np.lexsort((-np.arange(l.size), -l))")]),
+    "soft_mass_strict": ("soft_gate", "test_oracle_soft_gate", "osg",
+                         [("if a_ref and m >= rho:", "if a_ref and m > rho:")]),
+    "soft_empty_candidates_continue": ("soft_gate", "test_oracle_soft_gate", "osg",
+                                       [("if a_ref and m >= rho:", "if m >= rho and (a_ref or [None]):"),
+                                        ("a_star = a_ref[0]", "a_star = (a_ref or [int(np.argmax(l))])[0]")]),
     "soft_discard_step_late": ("soft_gate", "test_oracle_soft_gate", "osg",
                                [("st.decisive_step = st.steps\n", "st.decisive_step = st.steps + 1\n")]),
     "soft_softmax_unshifted_temperature": ("soft_gate", "test_oracle_soft_gate", "osg",

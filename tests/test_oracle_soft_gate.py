@@ -3,7 +3,8 @@
 Anchors: the appendix's worked illustration on a toy vocabulary
 (tests/golden/soft_gate_example.txt, outcomes worked out by hand), the limits
 that reduce it to the hard gate (K = 1, rho > 1, steps past the window c),
-and brute force over every compatible candidate.
+brute force over every compatible candidate, and the continue condition
+(m >= rho with a non-empty A_ref) at an exactly representable m.
 """
 import math
 import os
@@ -115,3 +116,21 @@ def test_top_k_ties_and_softmax():
     assert list(osg.top_k(l, 3)) == [1, 2, 4]
     p = osg.softmax(np.log(np.array([0.1, 0.2, 0.7])))
     assert np.allclose(p, [0.1, 0.2, 0.7], atol=1e-15)
+
+
+def test_mass_threshold_is_inclusive_and_needs_a_candidate():
+    # Alg. 2 goes on when m >= rho and A_ref is not empty.  Four equal logits give
+    # p = 1/4 exactly in fp64; the greedy token 0 leaves the refusal set, tokens 1
+    # and 2 keep it, so m = 1/2 exactly.
+    P = [[1, 3], [2, 3]]
+    logits = np.zeros(4)
+    st = ogate.GateState()
+    r = osg.soft_gate_step(st, logits, P, -1, 8, c=2, k=4, rho=0.5)
+    assert r.soft and r.mass == 0.5 and r.a_ref == [1, 2] and r.token == 1 and not st.done
+    st = ogate.GateState()
+    r = osg.soft_gate_step(st, logits, P, -1, 8, c=2, k=4, rho=float(np.nextafter(0.5, 1.0)))
+    assert r.soft and r.token is None and st.done and st.decision == ogate.NON_REFUSAL
+    # rho = 0 with no compatible token in the top K: A_ref is empty, so the probe ends
+    st = ogate.GateState()
+    r = osg.soft_gate_step(st, logits, P, -1, 8, c=2, k=1, rho=0.0)
+    assert r.soft and r.a_ref == [] and r.mass == 0.0 and r.token is None and st.done
