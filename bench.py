@@ -207,6 +207,35 @@ def clocks_rejected(clocks) -> bool:
     return bool(sm and smax and sm < 0.85 * smax and "sw_power_cap" not in reasons)
 
 
+def measure_with_clock_check(run_region, sync, clock, barrier=None, allreduce_max=None):
+    """Runs `run_region()` (the timed region) inside a clock sampler, bracketed
+    by `barrier` (all ranks) and `sync` (the device); when the clock record is
+    rejected on any rank (`allreduce_max` takes the max of a float over the
+    ranks), every rank runs the region once more.  Returns (the region's
+    result, the clock summary, whether it was measured again)."""
+    remeasured = False
+    for attempt in range(2):
+        if barrier is not None:
+            barrier()
+        sync()
+        with clock() as clk:
+            clk.start()
+            result = run_region()
+            sync()
+            clk.stop()
+        if barrier is not None:
+            barrier()
+        clocks = clk.summary()
+        redo = 1.0 if clocks_rejected(clocks) else 0.0
+        if allreduce_max is not None:
+            redo = allreduce_max(redo)  # every rank measures again, or none
+        if attempt == 0 and redo > 0:
+            remeasured = True
+            continue
+        break
+    return result, clocks, remeasured
+
+
 def _dist_env():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -380,28 +409,20 @@ def run_ours(args):
             split_step()
         torch.cuda.synchronize()
 
-    remeasured = False
-    for attempt in range(2):  # a region with a bad clock record is measured once more
-        if world > 1:
-            dist.barrier()
-        torch.cuda.synchronize()
-        with ClockSampler(torch.cuda.current_device()) as clk:
-            clk.start()
-            with torch.cuda.stream(stream):
-                step_ms = [one_step() for _ in range(args.steps)]
-                split = [split_step() for _ in range(args.steps)]
-            torch.cuda.synchronize()
-            clk.stop()
-        if world > 1:
-            dist.barrier()
-        clocks = clk.summary()
-        redo = torch.tensor([1.0 if clocks_rejected(clocks) else 0.0], dtype=torch.float64, device=dev)
-        if world > 1:
-            dist.all_reduce(redo, op=dist.ReduceOp.MAX)  # every rank measures again, or none
-        if attempt == 0 and float(redo.item()) > 0:
-            remeasured = True
-            continue
-        break
+    def timed_region():
+        with torch.cuda.stream(stream):
+            s_ms = [one_step() for _ in range(args.steps)]
+            sp = [split_step() for _ in range(args.steps)]
+        return s_ms, sp
+
+    def max_over_ranks(x: float) -> float:
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    (step_ms, split), clocks, remeasured = measure_with_clock_check(
+        timed_region, torch.cuda.synchronize, lambda: ClockSampler(torch.cuda.current_device()),
+        barrier=dist.barrier if world > 1 else None, allreduce_max=max_over_ranks if world > 1 else None)
     attn_ms = [t[0] for t in split]
     hg_ms = [t[1] for t in split]
     mean_step = sum(step_ms) / len(step_ms)

@@ -56,3 +56,57 @@ def test_rejection_rule():
     assert bench.clocks_rejected(dict(ok, sm_mhz=1200.0))                             # held low, no reason
     assert not bench.clocks_rejected(dict(ok, sm_mhz=1200.0, reasons=["sw_power_cap"]))
     assert not bench.clocks_rejected({"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"]})
+
+
+class FakeClock:
+    """Stands in for the nvidia-smi sampler: hands out prepared summaries."""
+
+    def __init__(self, records):
+        self.records = records
+
+    def __call__(self):
+        return self
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        return False
+
+    def start(self):
+        pass
+
+    def stop(self):
+        pass
+
+    def summary(self):
+        return dict(self.records.pop(0))
+
+
+GOOD = {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": []}
+THERMAL = {"sm_mhz": 1500.0, "sm_max_mhz": 2070.0, "reasons": ["hw_thermal_slowdown"]}
+
+
+def _region_counter():
+    runs = []
+
+    def region():
+        runs.append(len(runs))
+        return len(runs)
+    return region, runs
+
+
+def test_good_clock_record_is_measured_once():
+    region, runs = _region_counter()
+    res, clocks, again = bench.measure_with_clock_check(region, lambda: None, FakeClock([GOOD]))
+    assert runs == [0] and res == 1 and not again and clocks["sm_mhz"] == 2070.0
+
+
+def test_bad_clock_record_is_measured_once_more():
+    region, runs = _region_counter()
+    res, clocks, again = bench.measure_with_clock_check(region, lambda: None, FakeClock([THERMAL, GOOD]))
+    assert runs == [0, 1] and res == 2 and again and clocks["reasons"] == []
+    # a second bad record is kept (and reported): there is no third run
+    region, runs = _region_counter()
+    res, clocks, again = bench.measure_with_clock_check(region, lambda: None, FakeClock([THERMAL, THERMAL]))
+    assert runs == [0, 1] and again and clocks["reasons"] == ["hw_thermal_slowdown"]

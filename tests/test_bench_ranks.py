@@ -48,6 +48,49 @@ def test_two_gloo_ranks_agree_on_the_max():
         assert agg["value"] == 2 * 80 / 2e-3 and agg["e2e_value"] == 2 * 80 / 4e-3
 
 
+def _remeasure_worker(rank, world, port, out):
+    import torch
+    import torch.distributed as dist
+    sys.path.insert(0, ROOT)
+    sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))
+    import bench
+    from test_bench_clocks import GOOD, THERMAL, FakeClock
+    dist.init_process_group("gloo", init_method=f"tcp://127.0.0.1:{port}", rank=rank, world_size=world)
+    runs = []
+
+    def region():
+        runs.append(1)
+        return len(runs)
+
+    def max_over_ranks(x):
+        t = torch.tensor([x], dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    # only rank 1 sees a thermal slowdown; both ranks must run the region again
+    records = [THERMAL, GOOD] if rank == 1 else [GOOD, GOOD]
+    res, clocks, again = bench.measure_with_clock_check(region, lambda: None, FakeClock(records),
+                                                        barrier=dist.barrier, allreduce_max=max_over_ranks)
+    out.put((rank, len(runs), again))
+    dist.destroy_process_group()
+
+
+def test_a_bad_clock_on_one_rank_remeasures_every_rank():
+    pytest.importorskip("torch")
+    import torch.multiprocessing as mp
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_remeasure_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = dict((r, (n, a)) for r, n, a in (q.get(timeout=120) for _ in procs))
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    assert res == {0: (2, True), 1: (2, True)}
+
+
 def test_single_rank_needs_no_process_group():
     sys.path.insert(0, ROOT)
     import bench
