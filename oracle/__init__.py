@@ -16,6 +16,10 @@ Decoding") and the published definitions it relies on:
   sequences with the two-token minimum for token-prefix detections (App. D),
   as a naive scan over the refusal list, and the per-token hard-gate outcome of
   Alg. 1.
+* ``soft_gate``  -- one probe step of the soft compatibility gate of the
+  appendix ablation (Alg. 2): top-K, the compatible mass m against rho, a*.
+* ``precheck``   -- the residual-stream classifier of App. A: a d + 1 logistic
+  readout per prompt and the skip rule p <= theta, applied to the gate state.
 
 Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline /
 reference legs may import this package.  The product library never calls it and
@@ -23,5 +27,7 @@ shares no code with it; the two meet only through the seeded input generators.
 
 Parity status of each function is stated in its docstring; every function here
 is pinned by ``tests/test_oracle_*.py`` against closed forms, library routines,
-published known-answer vectors, brute force or the paper's worked examples.
+published known-answer vectors, brute force or the paper's worked examples,
+and ``tests/test_oracle_mutants.py`` checks that those pins catch plausible
+mistakes planted in copies of these modules.
 """
