@@ -40,6 +40,8 @@ MUTANTS = {
                                    [("kp = gather_tokens(k_pages, prompt_block_table[g], int(prompt_len[g]), h,",
                                      "kp = gather_tokens(k_pages, prompt_block_table[g], int(prompt_len[g]), "
                                      "(h + 1) % num_kv_heads,")]),
+    "attn_default_scale_1_over_d": ("attention", "test_oracle_attention", "attention",
+                                    [("scale = 1.0 / np.sqrt(D)", "scale = 1.0 / D")]),
     # ---- sample head ------------------------------------------------------------
     "samp_cutoff_sign": ("sampling", "test_oracle_sampling", "sampling",
                          [("theta32 = np.float32(t * np.log(m))", "theta32 = np.float32(-t * np.log(m))")]),
@@ -59,7 +61,11 @@ MUTANTS = {
                         'k = int(np.searchsorted(cdf, target, side="left"))')]),
     "samp_inactive_rows_sampled": ("sampling", "test_oracle_sampling", "sampling",
                                    [("        if not active[r]:\n            continue\n", "")]),
+    "samp_boundary_band_wide": ("sampling", "test_oracle_sampling", "sampling",
+                                [("BOUNDARY_REL = 1e-6", "BOUNDARY_REL = 1e-3")]),
     # ---- Philox4x32-10 ----------------------------------------------------------
+    "philox_product_halves_swapped": ("philox", "test_oracle_philox", "philox",
+                                      [("return p >> 32, p & MASK32", "return p & MASK32, p >> 32")]),
     "philox_weyl_constant": ("philox", "test_oracle_philox", "philox",
                              [("PHILOX_W1 = 0xBB67AE85", "PHILOX_W1 = 0xBB67AE84")]),
     "philox_high_halves_swapped": ("philox", "test_oracle_philox", "philox",
@@ -96,6 +102,11 @@ MUTANTS = {
                                   [("    if eos >= 0 and int(y) == eos:\n        st.done = True\n",
                                     "    if eos >= 0 and int(y) == eos:\n        st.q.append(int(y))\n"
                                     "        st.done = True\n")]),
+    "gate_confirm_needs_three": ("gate", "test_oracle_gate", "gate",
+                                 [("return any(len(pi) >= min_confirm and is_prefix(",
+                                   "return any(len(pi) > min_confirm and is_prefix(")]),
+    "gate_probe_row_left_on": ("gate", "test_oracle_gate", "gate",
+                               [("        if st.done:\n            out[g * rows_per_group] = 0\n", "")]),
     # ---- soft gate (Alg. 2) ---------------------------------------------------------
     "soft_mass_of_whole_top_k": ("soft_gate", "test_oracle_soft_gate", "osg",
                                  [("m = float(sum(p[a] for a in a_ref))", "m = float(sum(p[a] for a in top_k(l, k)))")]),
@@ -121,6 +132,8 @@ MUTANTS = {
     # ---- residual-stream precheck (App. A) ----------------------------------------
     "pre_bias_sign": ("precheck", "test_oracle_precheck", "precheck",
                       [("return h64 @ w64 + float(b)", "return h64 @ w64 - float(b)")]),
+    "pre_weights_reversed": ("precheck", "test_oracle_precheck", "precheck",
+                             [("return h64 @ w64 + float(b)", "return h64 @ w64[::-1] + float(b)")]),
     "pre_sigmoid_sign": ("precheck", "test_oracle_precheck", "precheck",
                          [("out[pos] = 1.0 / (1.0 + np.exp(-z[pos]))", "out[pos] = 1.0 / (1.0 + np.exp(z[pos]))")]),
     "pre_skip_strict": ("precheck", "test_oracle_precheck", "precheck",

@@ -99,6 +99,11 @@ def test_boundary_flag():
     # CDF steps at 0.25, 0.5, 1.0
     assert sampling.sample_from_uniform(row, 1.0, 0.0, 0.25).boundary
     assert not sampling.sample_from_uniform(row, 1.0, 0.0, 0.3).boundary
+    # the band is 1e-6 of Z on either side of a step: draws 5e-7 away are
+    # flagged, draws 2e-6 away are not
+    for du, flagged in ((5e-7, True), (-5e-7, True), (2e-6, False), (-2e-6, False)):
+        for step in (0.25, 0.5):
+            assert sampling.sample_from_uniform(row, 1.0, 0.0, step + du).boundary == flagged, (step, du)
 
 
 def test_temperature_to_zero_is_greedy():
