@@ -121,12 +121,16 @@ size_t rgd_prefix_decode_attn_workspace_size(const rgd_attn_shape* shape);
  *   out                bf16 [R, Hq, D]; lse float [R, Hq] or NULL
  *   workspace          device memory of rgd_prefix_decode_attn_workspace_size()
  *                      bytes, 256-byte aligned, zero-filled before its first
- *                      use.  It starts with one int32 counter per (group, kv
- *                      head) job, which every call leaves at zero again unless
- *                      it reports RGD_DEV_WAIT_TIMEOUT (then zero-fill it before
- *                      reuse); the rest is scratch that a call writes before
- *                      reading.  Calls that share a workspace must not overlap
- *                      in time.
+ *                      use.  It starts with an area of max(J, 8192) int32
+ *                      counters, J = num_groups * num_kv_heads (one per (group,
+ *                      kv head) job), which every call leaves at zero again
+ *                      unless it reports RGD_DEV_WAIT_TIMEOUT (then zero-fill it
+ *                      before reuse); the rest is scratch that a call writes
+ *                      before reading.  So one workspace, sized for the largest
+ *                      shape, may serve calls of any shapes with J <= 8192;
+ *                      a call with J > 8192 moves the scratch, so zero-fill the
+ *                      workspace whenever the shape changes across it.  Calls
+ *                      that share a workspace must not overlap in time.
  * One kernel runs on `stream`.  A job split across blocks is merged by the
  * block holding its first page, which waits (bounded) for the job's other
  * pieces; those are the first pieces of later blocks and wait on no other
@@ -154,13 +158,15 @@ int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf16* q,
  * or a latency-critical decode loop where cudaMalloc / cudaFree would
  * synchronise the device.  The caller still passes every input and output.
  *   - Shapes whose workspace (rgd_prefix_decode_attn_workspace_size) exceeds
- *     8 MiB are rejected with RGD_ERR_UNSUPPORTED.
+ *     8 MiB, or with more than 8192 (group, kv head) jobs, are rejected with
+ *     RGD_ERR_UNSUPPORTED.
  *   - The first call on a device looks up the array's device address (once per
  *     device, with that device current); make that first call before any stream
  *     capture.
  *   - Nothing is allocated or cleared: the array starts zeroed when the library
- *     is loaded and every call leaves its job counters at zero, unless it
- *     reports RGD_DEV_WAIT_TIMEOUT (after which this entry point must not be
+ *     is loaded; its first 32 KiB hold the job counters of every call, whatever
+ *     the shape, and every call leaves the counters of its jobs at zero, unless
+ *     it reports RGD_DEV_WAIT_TIMEOUT (after which this entry point must not be
  *     used again in the process).  Every call shares the one array, so calls
  *     that overlap on the GPU (other streams, other threads) race: serialise
  *     them. */

@@ -56,6 +56,7 @@
 // word and every role stops.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cmath>
 #include <mutex>
 
@@ -104,6 +105,7 @@ static_assert(kQCol + 64 <= 512, "TMEM columns");
 constexpr uint32_t kVLbo = 2048, kVSbo = 1024;
 constexpr float kRescaleLog2 = 8.f;           // lazy rescale threshold (factor 256)
 constexpr int kSmemLimit = 226 * 1024;        // dynamic part; static shared memory needs the rest
+constexpr int kTicketSlots = 8192;            // job counters at the start of every workspace (at least)
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
@@ -1366,8 +1368,12 @@ int make_plan(const rgd_attn_shape* s, Plan* pl) {
   pl->smem = layout(pl->nslots, pl->npref);
   auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
   const size_t n_part = (size_t)pl->C + pl->J - 1;  // partial-result slots
+  // The job counters come first, in an area of at least kTicketSlots counters
+  // whatever the shape, so that a workspace reused for another shape with up to
+  // kTicketSlots jobs finds its counters where earlier calls left zeros, not
+  // where they wrote partials.
   pl->ticket_off = 0;
-  pl->ml_off = up((size_t)pl->J * sizeof(int32_t));
+  pl->ml_off = up((size_t)std::max(pl->J, kTicketSlots) * sizeof(int32_t));
   pl->o_off = pl->ml_off + up(n_part * ml_stride(pl->nq) * sizeof(float2));
   pl->total = pl->o_off + up(n_part * pl->nq * s->head_dim * sizeof(float));
   return RGD_OK;
@@ -1505,6 +1511,12 @@ extern "C" int rgd_prefix_decode_attn_noalloc(const rgd_attn_shape* shape, const
                                               float* lse, int32_t* dev_status, rgd_stream_t stream) {
   clear_error();
   if (int rc = check_shape(shape)) return rc;
+  // The counters must sit in the fixed area at the start of the array for every
+  // shape (a larger job count would move the partials over them).
+  if ((int64_t)shape->num_groups * shape->num_kv_heads > kTicketSlots)
+    return set_error(RGD_ERR_UNSUPPORTED,
+                     "rgd_prefix_decode_attn_noalloc: num_groups * num_kv_heads = %lld exceeds %d",
+                     (long long)shape->num_groups * shape->num_kv_heads, kTicketSlots);
   const size_t need = ws_total(shape);
   if (need > kStaticScratchBytes)
     return set_error(RGD_ERR_UNSUPPORTED,
@@ -1529,7 +1541,8 @@ extern "C" int rgd_prefix_decode_attn_noalloc(const rgd_attn_shape* shape, const
     scratch = g_scratch_ptr[dev];
   }
   // the array is zero when the module is loaded (device variables without an
-  // initializer are zero-filled) and every call leaves its job counters at zero
+  // initializer are zero-filled); every call leaves the counters of its jobs at
+  // zero, and no call writes anything else into the fixed counter area
   return rgd_prefix_decode_attn(shape, q, k_pages, v_pages, prompt_block_table, prompt_len, suffix_block_table,
                                 suffix_len, row_active, softmax_scale, out, lse, scratch, kStaticScratchBytes,
                                 dev_status, stream);

@@ -13,6 +13,21 @@ def pytest_configure(config):
 
 import pytest  # noqa: E402
 
+_REPORT = []
+
+
+def report(line: str) -> None:
+    """Adds a line to the parity report printed at the end of the run (counts
+    of boundary rows and the like, shown without -s)."""
+    _REPORT.append(line)
+
+
+def pytest_terminal_summary(terminalreporter):
+    if _REPORT:
+        terminalreporter.write_sep("-", "parity report")
+        for line in _REPORT:
+            terminalreporter.write_line(line)
+
 
 @pytest.fixture(scope="session")
 def gpu_lib():

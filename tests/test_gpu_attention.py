@@ -74,17 +74,6 @@ def test_llama8b_other_block_counts(gpu_lib, ctas):
     _check(case, _run(case, num_ctas=ctas), rows=list(range(0, 80, 7)))
 
 
-def test_long_prompt_sampled_rows(gpu_lib):
-    case = workloads.long_prompt(seed=0).attn
-    _check(case, _run(case), rows=[0, 1, 13, 26, 35])
-
-
-def test_high_batch_sampled_rows(gpu_lib):
-    case = workloads.high_batch(seed=0).attn
-    inactive = [int(i) for i in np.nonzero(case.row_active == 0)[0][:3]]
-    _check(case, _run(case), rows=[0, 1, 2, 3, 100, 255, 256, 257, 510, 511] + inactive)
-
-
 def test_query_tiles_per_group(gpu_lib):
     # rows_per_group * Hq/Hkv = 1*4 (one tile), 3*8 (two query tiles), 16*8 = 128 (eight tiles)
     for rpg, Hq in [(1, 32), (3, 64), (16, 64)]:
