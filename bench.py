@@ -4,10 +4,13 @@
 One step = one pass of the whole hot path over one batch of the Llama-3-8B-shaped
 workload (16 prompts x (1 greedy probe + 4 high-temperature sample rows), prompts
 U[512, 2048] tokens, suffixes U[0, 256], 32 q / 8 kv heads, head dim 128, bf16 KV
-in 16-token pages, fp32 logits over 128256): shared-prefix split-KV attention,
-the sample head (argmax / temperature + min-p + Philox draw) and the trie gate.
-Inputs are seeded synthetic data resident in HBM; L2 is flushed (256 MiB write)
-before every timed step, outside the timed events.
+in 16-token pages, fp32 logits over 128256): one rgd_decode_step, i.e. the
+shared-prefix split-KV attention, then the sample head (argmax / temperature +
+min-p + Philox draw) with the trie gate fused in.  Inputs are seeded synthetic
+data resident in HBM; L2 is evicted (a 256 MiB write, then a 320 MiB read)
+before every timed step, outside the timed events.  Extra keys time the
+long-prompt and high-batch steps, the largest head and gate sweeps, the whole
+128-step gated loop, the soft gate and the residual precheck.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -322,6 +325,236 @@ def run_reference(args):
 # ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
+class Evictor:
+    """Empties L2 of the next timed call's inputs, outside the timed events: a
+    256 MiB write, then a read of 320 MiB (more than twice the 129 MB L2), so
+    that the lines left in L2 are clean and the timed call pays no write-back
+    of the eviction traffic.  ``clean=False`` stops after the write (then up
+    to an L2 of dirty lines is written back inside the timed region)."""
+
+    def __init__(self, dev):
+        import torch
+        self.w = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+        self.r = torch.ones((320 << 20) // 8, dtype=torch.int64, device=dev)
+        self.sink = torch.empty((), dtype=torch.int64, device=dev)
+
+    def __call__(self, clean: bool = True):
+        import torch
+        self.w.fill_(1)
+        if clean:
+            torch.sum(self.r, dim=0, out=self.sink)
+
+
+class StepOnDevice:
+    """One decode step's buffers on the device and its calls: rgd_decode_step
+    (attention, then the sample head with the gate fused in), its two halves
+    apart, and the reset of the state the gate changes (gate states and row
+    mask back to the step's start), run outside the timed events."""
+
+    def __init__(self, case, dev, kv=None):
+        import torch
+        from paper_2607_20791_gb300 import binding, device
+        self.case = case
+        self.att = device.attn_to_device(case.attn, device=dev, kv=kv)
+        self.head = device.head_to_device(case.head, device=dev)
+        self.trie = binding.Trie(case.gate.refusal_seqs, case.gate.min_confirm)
+        self.G, self.rpg = case.attn.num_groups, case.attn.rows_per_group
+        self.gstate = binding.new_gate_state(self.G, device=dev)
+        self.ra0 = self.att.row_active.clone()
+        self.status = torch.zeros(1, dtype=torch.int32, device=dev)
+
+    def reset(self, s):
+        from paper_2607_20791_gb300 import binding
+        binding.rgd_gate_state_init(self.gstate, self.G, stream=s)
+        self.att.row_active.copy_(self.ra0)
+
+    def step(self, s):
+        from paper_2607_20791_gb300 import binding
+        a, h, g = self.att, self.head, self.case.gate
+        binding.rgd_decode_step(a.shape, a.q, a.k_pages, a.v_pages, a.prompt_block_table, a.prompt_len,
+                                a.suffix_block_table, a.suffix_len, a.softmax_scale, a.out, a.lse, a.workspace,
+                                h.logits, h.is_probe, h.temperature, h.min_p, h.seed, h.step, a.row_active,
+                                h.token_out, h.kept_count, self.trie, g.eos, g.max_len, self.gstate, self.status,
+                                stream=s)
+
+    def attn(self, s):
+        from paper_2607_20791_gb300 import binding
+        a = self.att
+        binding.rgd_prefix_decode_attn(a.shape, a.q, a.k_pages, a.v_pages, a.prompt_block_table, a.prompt_len,
+                                       a.suffix_block_table, a.suffix_len, a.row_active, a.softmax_scale, a.out,
+                                       a.lse, a.workspace, self.status, stream=s)
+
+    def head_gate(self, s):
+        from paper_2607_20791_gb300 import binding
+        a, h, g = self.att, self.head, self.case.gate
+        binding.rgd_sample_head_gated(h.logits, h.is_probe, h.temperature, h.min_p, h.seed, h.step, a.row_active,
+                                      h.token_out, h.kept_count, self.trie, self.rpg, g.eos, g.max_len,
+                                      self.gstate, self.status, stream=s)
+
+    def close(self):
+        self.trie.close()
+
+
+def _median(xs):
+    xs = sorted(xs)
+    return xs[len(xs) // 2]
+
+
+def time_step(sd, stream, evict, n, warmup=3):
+    """Graph of one step (timed with events around each replay, L2 evicted and
+    state reset before each), then the same number of eager steps with events
+    around attention and around the gated head.  Means in ms."""
+    import torch
+    s = stream.cuda_stream
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            sd.reset(s)
+            sd.step(s)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            sd.step(s)
+        torch.cuda.synchronize()
+        step_ms, attn_ms, head_ms = [], [], []
+        for i in range(warmup + n):
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+            evict()
+            sd.reset(s)
+            ev[0].record(stream)
+            g.replay()
+            ev[1].record(stream)
+            ev[1].synchronize()
+            if i >= warmup:
+                step_ms.append(ev[0].elapsed_time(ev[1]))
+        for i in range(warmup + n):
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+            evict()
+            sd.reset(s)
+            ev[0].record(stream)
+            sd.attn(s)
+            ev[1].record(stream)
+            sd.head_gate(s)
+            ev[2].record(stream)
+            ev[2].synchronize()
+            if i >= warmup:
+                attn_ms.append(ev[0].elapsed_time(ev[1]))
+                head_ms.append(ev[1].elapsed_time(ev[2]))
+    mean = lambda x: sum(x) / len(x)
+    return g, mean(step_ms), mean(attn_ms), mean(head_ms)
+
+
+def _device_kv(attn_case, dev, seed):
+    """K and V pools ~ N(0, 1) in bf16, drawn on the device (the kernels' time
+    does not depend on the values; the parity tests use the seeded host draw)."""
+    import torch
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(seed)
+    shape = (attn_case.num_pages, attn_case.num_kv_heads, attn_case.page_size, attn_case.head_dim)
+    k = torch.randn(shape, generator=gen, device=dev, dtype=torch.bfloat16)
+    v = torch.randn(shape, generator=gen, device=dev, dtype=torch.bfloat16)
+    return k, v
+
+
+def config_leg(name, case, dev, stream, evict, n, peak):
+    """Throughput and HBM roofline fraction of one more configuration's step."""
+    import torch
+    sd = StepOnDevice(case, dev, kv=_device_kv(case.attn, dev, seed=7))
+    _, step_ms, attn_ms, head_ms = time_step(sd, stream, evict, n)
+    attn_b, head_b = algorithmic_bytes(case)
+    status = int(sd.status.item())
+    rows = int(case.head.row_active.sum())
+    sd.close()
+    del sd
+    torch.cuda.empty_cache()
+    gbs = lambda b, ms: b / (ms / 1e3) / 1e9
+    return {"workload": name, "rows_per_step": rows, "ms_per_step": step_ms, "rows_per_s": rows / (step_ms / 1e3),
+            "attention_ms": attn_ms, "head_gate_ms": head_ms, "attention_bytes": attn_b, "logits_bytes": head_b,
+            "step_hbm_frac": gbs(attn_b + head_b, step_ms) / peak,
+            "attention_hbm_frac": gbs(attn_b, attn_ms) / peak,
+            "head_hbm_frac": gbs(head_b, head_ms) / peak, "dev_status": status}
+
+
+def sweep_leg(dev, stream, evict, n, peak):
+    """The largest head sweep (1024 x 262144, fp32 and bf16; temperatures
+    0-10, min-p 0-0.3) and the gate sweep (1024 groups, 1000 refusal
+    sequences, 32-token probes), each kernel timed alone."""
+    import torch
+    from paper_2607_20791_gb300 import binding, device, workloads
+    out = {}
+    base = workloads.head_sweep(1024, 262144, "f32", seed=11)
+    for dt in ("f32", "bf16"):
+        hc = base if dt == "f32" else workloads.make_head_case(
+            base.name, base.logits, "bf16", base.is_probe, base.temperature, base.min_p, seed=11)
+        h = device.head_to_device(hc, device=dev)
+        ts = []
+        with torch.cuda.stream(stream):
+            for i in range(3 + n):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                evict()
+                e0.record(stream)
+                h.run(stream=stream.cuda_stream, with_mask=False)
+                e1.record(stream)
+                e1.synchronize()
+                if i >= 3:
+                    ts.append(e0.elapsed_time(e1))
+        b = hc.rows * hc.vocab * (4 if dt == "f32" else 2)
+        ms = sum(ts) / len(ts)
+        out[f"head_1024x262144_{dt}"] = {"us": 1e3 * ms, "bytes": b, "hbm_frac": b / (ms / 1e3) / 1e9 / peak,
+                                          "dev_status": int(h.dev_status.item())}
+        del h
+    gc = workloads.gate_sweep(groups=1024, n_seq=1000, vocab=128256, n_steps=32, seed=3)
+    trie = binding.Trie(gc.refusal_seqs, 2)
+    st = binding.new_gate_state(1024, device=dev)
+    toks = torch.from_numpy(gc.tokens).to(dev)
+    ts = []
+    with torch.cuda.stream(stream):
+        for i in range(3 + n):
+            binding.rgd_gate_state_init(st, 1024, stream=stream.cuda_stream)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            binding.rgd_probe_gate(trie, 1024, 1, toks, 32, 32, gc.eos, gc.max_len, st, stream=stream.cuda_stream)
+            e1.record(stream)
+            e1.synchronize()
+            if i >= 3:
+                ts.append(e0.elapsed_time(e1))
+    trie.close()
+    out["gate_1024x32_tokens"] = {"us": 1e3 * sum(ts) / len(ts), "note": "32 probe tokens per group in one call"}
+    torch.cuda.empty_cache()
+    return out
+
+
+def loop_leg(dev, stream, evict, n):
+    """The Llama-3-8B-shaped gated loop (128 steps from the prompt end, one CUDA
+    graph; per step the probe tokens are planted in the logits, one
+    rgd_decode_step runs, the logits go back and the active rows' suffixes
+    grow): time per loop and active rows per second."""
+    import torch
+    from paper_2607_20791_gb300 import device, workloads
+    case = workloads.llama8b_loop(seed=0, with_kv=False)
+    case.attn.k_pages, case.attn.v_pages = None, None
+    kv = _device_kv(case.attn, dev, seed=8)
+    loop = device.DeviceLoop(case, stream, keep_history=False, kv=kv)
+    loop.capture()
+    ts = []
+    with torch.cuda.stream(stream):
+        for i in range(2 + n):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            evict()
+            e0.record(stream)
+            loop.graph.replay()
+            e1.record(stream)
+            e1.synchronize()
+            if i >= 2:
+                ts.append(e0.elapsed_time(e1))
+    rows = int((loop.tok >= 0).sum().item())  # rows that drew a token, over the loop's steps
+    status = int(loop.status.item())
+    loop.close()
+    ms = sum(ts) / len(ts)
+    return {"steps": case.n_steps, "ms_per_loop": ms, "us_per_step": 1e3 * ms / case.n_steps,
+            "active_rows_per_loop": rows, "rows_per_s": rows / (ms / 1e3), "dev_status": status,
+            "launches_per_step": {"library": 2, "torch (input staging, suffix growth)": 3}}
+
+
 def run_ours(args):
     import torch
     world, rank, local = _dist_env()
@@ -335,56 +568,39 @@ def run_ours(args):
 
     import __graft_entry__
     __graft_entry__.build()
-    from paper_2607_20791_gb300 import binding, device, workloads
+    from paper_2607_20791_gb300 import binding, workloads
 
+    peak, peak_kind = _peaks()
     case = workloads.llama8b(seed=rank)
     attn_bytes, head_bytes = algorithmic_bytes(case)
     step_bytes = attn_bytes + head_bytes
     G, rpg = case.attn.num_groups, case.attn.rows_per_group
     R = G * rpg
     rows_per_step = int(case.head.row_active.sum())
-
-    att = device.attn_to_device(case.attn, device=dev)
-    head = device.head_to_device(case.head, device=dev)
-    trie = binding.Trie(case.gate.refusal_seqs, 2)
-    gstate = binding.new_gate_state(G, device=dev)
-    gate_active = torch.ones(R, dtype=torch.uint8, device=dev)
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     stream = torch.cuda.Stream(device=dev)
+    s = stream.cuda_stream
+    evict = Evictor(dev)
+    sd = StepOnDevice(case, dev)
 
-    def attn_call():
-        att.run(stream=stream.cuda_stream)
-
-    def head_gate_call():
-        binding.rgd_sample_head(head.logits, head.is_probe, head.temperature, head.min_p, head.seed, head.step,
-                                head.row_active, head.token_out, head.kept_count, None, head.dev_status,
-                                stream=stream.cuda_stream)
-        # the gate runs on the probe rows' tokens; its state is reset each step so
-        # every step gates the same first probe token (the step is timed alone)
-        binding.rgd_gate_state_init(gstate, G, stream=stream.cuda_stream)
-        binding.rgd_probe_gate(trie, G, rpg, head.token_out, 1, rpg, case.gate.eos, case.gate.max_len, gstate,
-                               gate_active, head.dev_status, stream=stream.cuda_stream)
-
-    # The whole step is one CUDA graph (the headline is timed on it).  The split
-    # into attention and sample head + gate comes from a second pass of the same
-    # steps launched eagerly, with events around each part: an event recorded
-    # inside the graph would itself leave the GPU idle for ~5 us per step.
+    # The step is one CUDA graph of rgd_decode_step (two kernels: attention,
+    # then the gated head, scheduled while the attention finishes); the headline
+    # is timed on it.  The split into attention and gated head comes from a
+    # second pass of as many steps launched eagerly with events around each.
     with torch.cuda.stream(stream):
         for _ in range(3):  # eager warm-up (also sets kernel attributes before capture)
-            attn_call()
-            head_gate_call()
+            sd.reset(s)
+            sd.step(s)
         torch.cuda.synchronize()
         g_step = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g_step, stream=stream):
-            attn_call()
-            head_gate_call()
+            sd.step(s)
         torch.cuda.synchronize()
-    launches_per_step = 4  # attention (split jobs merged inside), sample head, gate-state reset, gate
+    launches_per_step = 2  # attention (split jobs merged inside), sample head with the gate fused in
 
     def one_step():
-        """Runs one timed step (the graph); returns its time in ms."""
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
-        flush.fill_(1)
+        evict()
+        sd.reset(s)
         ev[0].record(stream)
         g_step.replay()
         ev[1].record(stream)
@@ -392,13 +608,13 @@ def run_ours(args):
         return ev[0].elapsed_time(ev[1])
 
     def split_step():
-        """Runs one step eagerly; returns (attention, head + gate) in ms."""
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
-        flush.fill_(1)
+        evict()
+        sd.reset(s)
         ev[0].record(stream)
-        attn_call()
+        sd.attn(s)
         ev[1].record(stream)
-        head_gate_call()
+        sd.head_gate(s)
         ev[2].record(stream)
         ev[2].synchronize()
         return ev[0].elapsed_time(ev[1]), ev[1].elapsed_time(ev[2])
@@ -427,10 +643,29 @@ def run_ours(args):
     hg_ms = [t[1] for t in split]
     mean_step = sum(step_ms) / len(step_ms)
     mean_attn = sum(attn_ms) / len(attn_ms)
-    status = int(att.dev_status.item()) | int(head.dev_status.item())
+    mean_hg = sum(hg_ms) / len(hg_ms)
+    status = int(sd.status.item())
+    n_side = max(5, min(args.steps, 100))  # steps of the legs outside the headline
+
+    # ---- the attention after a write-only eviction: the dirty lines it leaves
+    # in L2 are written back inside the timed region (context for the headline's
+    # clean eviction)
+    dirty_ms, clean_ms = [], []
+    with torch.cuda.stream(stream):
+        for i in range(3 + n_side):
+            for clean, acc in ((False, dirty_ms), (True, clean_ms)):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                evict(clean=clean)
+                sd.reset(s)
+                e0.record(stream)
+                sd.attn(s)
+                e1.record(stream)
+                e1.synchronize()
+                if i >= 3:
+                    acc.append(e0.elapsed_time(e1))
 
     # ---- the residual-stream precheck (App. A): once per prompt, not per step;
-    # timed alone on the step's 16 groups (d = 4096 bf16), L2 flushed before each
+    # timed alone on the step's 16 groups (d = 4096 bf16)
     pre = workloads.llama8b_precheck(seed=rank)
     pre_h = torch.from_numpy(pre.h.view(np.int16)).to(dev).view(torch.bfloat16)
     pre_w = torch.from_numpy(pre.w).to(dev)
@@ -438,94 +673,140 @@ def run_ours(args):
     pre_prob = torch.empty(G, dtype=torch.float32, device=dev)
     pre_ms = []
     with torch.cuda.stream(stream):
-        for i in range(args.warmup + args.steps):
-            binding.rgd_gate_state_init(pre_st, G, stream=stream.cuda_stream)
-            flush.fill_(1)
+        for i in range(3 + n_side):
+            binding.rgd_gate_state_init(pre_st, G, stream=s)
+            evict()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-            binding.rgd_residual_precheck(pre_h, pre_w, pre.b, pre.theta, rpg, pre_st, None, pre_prob,
-                                          stream=stream.cuda_stream)
+            binding.rgd_residual_precheck(pre_h, pre_w, pre.b, pre.theta, rpg, pre_st, None, pre_prob, stream=s)
             e1.record(stream)
             e1.synchronize()
-            if i >= args.warmup:
+            if i >= 3:
                 pre_ms.append(e0.elapsed_time(e1))
     pre_bytes = pre.groups * pre.d * 2 + pre.d * 4 + pre.groups * (4 + 20)
 
     # ---- the soft compatibility gate (the appendix ablation's Alg. 2): an
     # alternative to the hard gate; timed alone on the step's probe rows from a
     # fresh state (top-K 40, rho 0.1; the step's greedy tokens mostly leave the
-    # refusal set, so the soft branch runs), L2 flushed before each call
+    # refusal set, so the soft branch runs)
+    head = sd.head
     soft_tok = torch.empty(G, dtype=torch.int32, device=dev)
     soft_ms = []
     with torch.cuda.stream(stream):
-        for i in range(args.warmup + args.steps):
-            binding.rgd_gate_state_init(pre_st, G, stream=stream.cuda_stream)
-            flush.fill_(1)
+        for i in range(3 + n_side):
+            binding.rgd_gate_state_init(pre_st, G, stream=s)
+            evict()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-            binding.rgd_soft_gate(trie, G, rpg, head.logits, rpg * head.logits.shape[1], 40, 0.1, 8,
-                                  case.gate.eos, case.gate.max_len, pre_st, soft_tok, stream=stream.cuda_stream)
+            binding.rgd_soft_gate(sd.trie, G, rpg, head.logits, rpg * head.logits.shape[1], 40, 0.1, 8,
+                                  case.gate.eos, case.gate.max_len, pre_st, soft_tok, stream=s)
             e1.record(stream)
             e1.synchronize()
-            if i >= args.warmup:
+            if i >= 3:
                 soft_ms.append(e0.elapsed_time(e1))
     soft_bytes = G * head.logits.shape[1] * head.logits.element_size()
 
     # ---- end to end through the public API with host buffers ----------------
-    h2d_src = {
-        "q": case.attn.q, "logits": case.head.logits, "prompt_block_table": case.attn.prompt_block_table,
-        "prompt_len": case.attn.prompt_len, "suffix_block_table": case.attn.suffix_block_table,
-        "suffix_len": case.attn.suffix_len, "row_active": case.attn.row_active,
-        "temperature": case.head.temperature, "min_p": case.head.min_p, "seed": case.head.seed.view(np.int64),
-        "is_probe": case.head.is_probe}
-    dst = {"q": att.q, "logits": head.logits, "prompt_block_table": att.prompt_block_table,
-           "prompt_len": att.prompt_len, "suffix_block_table": att.suffix_block_table,
-           "suffix_len": att.suffix_len, "row_active": att.row_active, "temperature": head.temperature,
-           "min_p": head.min_p, "seed": head.seed, "is_probe": head.is_probe}
-    pinned = {}
-    for k, a in h2d_src.items():
-        t = torch.from_numpy(np.ascontiguousarray(a))
-        if dst[k].dtype != t.dtype:
-            t = t.view(dst[k].dtype)
-        pinned[k] = t.reshape(dst[k].shape).pin_memory()
-    h2d_bytes = sum(t.numel() * t.element_size() for t in pinned.values())
+    # One CUDA graph per step: the head's inputs (41 MB of logits) are copied on
+    # a second stream while the attention's inputs are copied and the attention
+    # runs; the gated head waits for both; the tokens and gate states are read
+    # back.  Every input comes from pinned host memory each step.
+    att = sd.att
+    attn_src = {"q": (case.attn.q, att.q), "prompt_block_table": (case.attn.prompt_block_table, att.prompt_block_table),
+                "prompt_len": (case.attn.prompt_len, att.prompt_len),
+                "suffix_block_table": (case.attn.suffix_block_table, att.suffix_block_table),
+                "suffix_len": (case.attn.suffix_len, att.suffix_len), "row_active": (case.attn.row_active, att.row_active)}
+    head_src = {"logits": (case.head.logits, head.logits), "temperature": (case.head.temperature, head.temperature),
+                "min_p": (case.head.min_p, head.min_p), "seed": (case.head.seed.view(np.int64), head.seed),
+                "is_probe": (case.head.is_probe, head.is_probe)}
+
+    def pin(src):
+        out = {}
+        for k, (a, d) in src.items():
+            t = torch.from_numpy(np.ascontiguousarray(a))
+            if d.dtype != t.dtype:
+                t = t.view(d.dtype)
+            out[k] = (t.reshape(d.shape).pin_memory(), d)
+        return out
+
+    attn_pin, head_pin = pin(attn_src), pin(head_src)
+    h2d_bytes = sum(t.numel() * t.element_size() for t, _ in list(attn_pin.values()) + list(head_pin.values()))
     tok_host = torch.empty(R, dtype=torch.int32).pin_memory()
-    st_host = torch.empty_like(gstate, device="cpu").pin_memory()
+    st_host = torch.empty_like(sd.gstate, device="cpu").pin_memory()
     d2h_bytes = tok_host.numel() * 4 + st_host.numel()
-    e2e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-              for _ in range(args.steps)]
+    side = torch.cuda.Stream(device=dev)
+
+    def e2e_body():
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            for t, d in head_pin.values():
+                d.copy_(t, non_blocking=True)
+        for t, d in attn_pin.values():
+            d.copy_(t, non_blocking=True)
+        sd.attn(s)
+        stream.wait_stream(side)
+        sd.head_gate(s)
+        tok_host.copy_(head.token_out, non_blocking=True)
+        st_host.copy_(sd.gstate, non_blocking=True)
+
     with torch.cuda.stream(stream):
-        for i in range(args.warmup + args.steps):
-            flush.fill_(1)
-            if i >= args.warmup:
-                e2e_ev[i - args.warmup][0].record(stream)
-            for k, t in pinned.items():
-                dst[k].copy_(t, non_blocking=True)
-            g_step.replay()
-            tok_host.copy_(head.token_out, non_blocking=True)
-            st_host.copy_(gstate, non_blocking=True)
-            if i >= args.warmup:
-                e2e_ev[i - args.warmup][1].record(stream)
+        sd.reset(s)
+        e2e_body()
         torch.cuda.synchronize()
-    e2e_ms = sum(a.elapsed_time(b) for a, b in e2e_ev) / args.steps
+        g_e2e = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_e2e, stream=stream):
+            e2e_body()
+        torch.cuda.synchronize()
+        e2e_list = []
+        for i in range(args.warmup + args.steps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            evict()
+            binding.rgd_gate_state_init(sd.gstate, G, stream=s)
+            e0.record(stream)
+            g_e2e.replay()
+            e1.record(stream)
+            e1.synchronize()
+            if i >= args.warmup:
+                e2e_list.append(e0.elapsed_time(e1))
+    e2e_ms = sum(e2e_list) / len(e2e_list)
 
     # ---- size-matched copy (context for the roofline fraction) ------------------
     # a plain device copy moving the attention's algorithmic byte count (half read,
-    # half written), L2 flushed before each, timed with events like the kernels:
-    # the bandwidth a transfer of this size reaches at all
+    # half written), timed like the kernels after each eviction: the bandwidth a
+    # transfer of this size reaches at all
     half = (attn_bytes // 2 + 15) // 16 * 16
     c_src = torch.ones(half, dtype=torch.uint8, device=dev)
     c_dst = torch.empty_like(c_src)
-    c_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(12)]
+    copy_res = {}
     with torch.cuda.stream(stream):
-        for a, b in c_ev:
-            flush.fill_(1)
-            a.record(stream)
-            c_dst.copy_(c_src)
-            b.record(stream)
-    torch.cuda.synchronize()
-    copy_ms = sorted(a.elapsed_time(b) for a, b in c_ev[3:])[4]
+        for clean in (True, False):
+            ts = []
+            for i in range(12):
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                evict(clean=clean)
+                a.record(stream)
+                c_dst.copy_(c_src)
+                b.record(stream)
+                b.synchronize()
+                if i >= 3:
+                    ts.append(a.elapsed_time(b))
+            copy_res[clean] = _median(ts)
     del c_src, c_dst
+    copy_ms = copy_res[True]
+
+    # ---- the other configurations (rank 0 only: extra keys, not the headline)
+    legs = {}
+    if rank == 0:
+        legs["long_prompt"] = config_leg(
+            "4 prompts x 32768 tokens, 1 probe + 8 sample rows, suffix U[0,1024], 64 q / 8 kv heads, D 128, "
+            "bf16 logits over 128256, T 2, min-p 0.05", workloads.long_prompt(seed=0, with_kv=False), dev, stream,
+            evict, n_side, peak)
+        legs["high_batch"] = config_leg(
+            "256 prompts, lengths log-normal (median 1024, sigma 1, 128-8192), 1 probe + 1 sample row, 30 % of "
+            "groups' sample rows off, 32 q / 8 kv heads, D 128, bf16 logits over 152064",
+            workloads.high_batch(seed=0, with_kv=False), dev, stream, evict, n_side, peak)
+        legs["sweep"] = sweep_leg(dev, stream, evict, n_side, peak)
+        legs["gated_loop"] = loop_leg(dev, stream, evict, max(3, min(args.steps, 10)))
 
     # ---- max over ranks --------------------------------------------------------
     agg = aggregate_over_ranks(mean_step, e2e_ms, mean_attn, rows_per_step, world, device=dev)
@@ -533,7 +814,6 @@ def run_ours(args):
     value, e2e_value = agg["value"], agg["e2e_value"]
 
     if rank == 0:
-        peak, peak_kind = _peaks()
         attn_gbs = attn_bytes / (mean_attn / 1e3) / 1e9
         step_gbs = step_bytes / (mean_step / 1e3) / 1e9
         traffic = _profiled_traffic()
@@ -544,37 +824,51 @@ def run_ours(args):
             "warmup": args.warmup, "ms_per_step": mean_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": WORKLOAD, "rows_per_step": rows_per_step, "groups": G,
-                       "l2": "flushed between steps (256 MiB write, outside the timed events)",
-                       "timing": "CUDA events per step on the launching stream around one CUDA graph of the "
-                                 "step (attention, sample head, gate); kernels_ms and roofline from a second "
-                                 "pass of as many steps launched eagerly with events around each part",
+                       "l2": "evicted before every timed step, outside the timed events: a 256 MiB write, then a "
+                             "320 MiB read, so that L2 holds only clean lines of other data",
+                       "timing": "CUDA events per step on the launching stream around one CUDA graph of "
+                                 "rgd_decode_step (attention, then the sample head with the gate fused in); gate "
+                                 "states and row mask reset before each step outside the events; kernels_ms and "
+                                 "roofline from a second pass of as many steps launched eagerly with events around "
+                                 "each kernel",
                        "parallelism": f"replicas x{world}"},
             "step_hbm_gbs": step_gbs, "step_hbm_frac": step_gbs / peak,
             "step_algorithmic_bytes": step_bytes,
-            "kernels_ms": {"attention": mean_attn, "sample_head_and_gate": sum(hg_ms) / len(hg_ms)},
+            "kernels_ms": {"attention": mean_attn, "sample_head_with_gate": mean_hg},
             "roofline": {"bound": "hbm", "kernel": "attn_tc_kernel<128, 4>", "achieved": attn_gbs,
                          "peak": peak, "unit": "GB/s", "frac": attn_gbs / peak, "traffic": traffic,
+                         "traffic_source": ("ncu capture of this kernel source (dram bytes read + written per "
+                                            "launch), recorded in profiles/attn_tc_kernel_llama8b.md"
+                                            if traffic is not None else
+                                            "none: no ncu capture of the current kernel source"),
                          "algorithmic_bytes": attn_bytes, "peak_source": peak_kind},
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
-                    "d2h_bytes_per_step": d2h_bytes, "ms_per_step": e2e_ms},
+                    "d2h_bytes_per_step": d2h_bytes, "ms_per_step": e2e_ms,
+                    "note": "one CUDA graph per step: logits and head inputs copied on a second stream while the "
+                            "attention inputs are copied and the attention runs"},
             "gpu_launches": launches_per_step * args.steps,
             "split_pass_launches": launches_per_step * args.steps,
-            "soft_gate": {"us": 1e3 * sorted(soft_ms)[len(soft_ms) // 2], "groups": G,
-                          "bytes": soft_bytes, "gbs": soft_bytes / (sorted(soft_ms)[len(soft_ms) // 2] / 1e3) / 1e9,
+            "attention_after_write_only_eviction_ms": sum(dirty_ms) / len(dirty_ms),
+            "attention_after_clean_eviction_ms": sum(clean_ms) / len(clean_ms),
+            "soft_gate": {"us": 1e3 * _median(soft_ms), "groups": G, "bytes": soft_bytes,
+                          "gbs": soft_bytes / (_median(soft_ms) / 1e3) / 1e9,
                           "note": "alternative to the hard gate (top-K 40, rho 0.1), outside the step"},
-            "residual_precheck": {"us": 1e3 * sorted(pre_ms)[len(pre_ms) // 2], "groups": pre.groups, "d": pre.d,
+            "residual_precheck": {"us": 1e3 * _median(pre_ms), "groups": pre.groups, "d": pre.d,
                                   "bytes": pre_bytes, "bound": "launch latency (a d + 1 logistic readout)",
                                   "note": "once per prompt, outside the step"},
             "copy_ceiling": {"bytes": 2 * half, "us": copy_ms * 1e3, "gbs": 2 * half / (copy_ms / 1e3) / 1e9,
                              "frac_of_peak": 2 * half / (copy_ms / 1e3) / 1e9 / peak,
                              "attention_frac_of_copy": copy_ms / mean_attn,
+                             "after_write_only_eviction_us": copy_res[False] * 1e3,
                              "note": "a plain device copy of the attention's algorithmic byte count (half read, "
-                                     "half written), L2 flushed, median of 9: what a transfer of this size reaches"},
+                                     "half written), L2 evicted as for the step, median of 9: what a transfer of "
+                                     "this size reaches"},
+            "configs": legs,
             "clocks": clocks, "dev_status": status,
         }
         print(json.dumps(line), flush=True)
-    trie.close()
+    sd.close()
     if world > 1:
         dist.destroy_process_group()
 

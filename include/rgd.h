@@ -14,6 +14,8 @@
  *   rgd_prefix_decode_attn  shared-prefix split-KV decode attention,
  *   rgd_sample_head         greedy argmax / temperature + min-p + Philox sample,
  *   rgd_probe_gate          per-token refusal-prefix gate on a token trie,
+ *   rgd_sample_head_gated   the two above in one kernel,
+ *   rgd_decode_step         attention, then the gated head: one whole step,
  *   rgd_soft_gate           its soft variant (the appendix ablation, Alg. 2),
  *   rgd_residual_precheck   the residual-stream classifier that lets a prompt
  *                           skip the probe (App. A), once per prompt.
@@ -93,6 +95,15 @@ typedef struct {
   int32_t num_ctas;          /* persistent blocks (<= 65535); 0 = one per SM     */
   int32_t reserved;          /* must be 0                                       */
 } rgd_attn_shape;
+
+/* Sets how long the attention kernel's blocks wait for one another (a split
+ * job's merger for its other pieces) and for their own copies and MMAs before
+ * giving up with RGD_DEV_WAIT_TIMEOUT, for every later call on any thread; 0
+ * restores the default of 2 s.  The kernel never traps: a wait that gives up
+ * stops that block's work, drains its copies in flight and returns.  A short
+ * limit serves tests of that path; in service a limit must stay far above a
+ * call's run time. */
+int rgd_set_wait_limit_ns(uint64_t limit_ns);
 
 /* Bytes of device workspace rgd_prefix_decode_attn needs for this shape (it
  * depends on the current device's SM count when num_ctas is 0). */
@@ -233,7 +244,7 @@ typedef struct {
   uint8_t decision;       /* RGD_PENDING / RGD_REFUSAL / RGD_NON_REFUSAL             */
   uint8_t confirmed;      /* some refusal prefix of length >= min_confirm prefixes q */
   uint8_t done;           /* the probe has ended (stop token, length cap, discarded) */
-  uint8_t reserved;
+  uint8_t reserved;       /* 0 between calls (rgd_sample_head_gated counts rows here) */
 } rgd_gate_state;
 
 /* Reset `groups` states to the empty probe (node 0, pending). */
@@ -258,6 +269,52 @@ int rgd_probe_gate(const rgd_trie* trie, int32_t groups, int32_t rows_per_group,
                    const int32_t* probe_tokens, int32_t n_tokens, int64_t token_stride,
                    int32_t eos_token, int32_t max_len, rgd_gate_state* state,
                    uint8_t* row_active, int32_t* dev_status, rgd_stream_t stream);
+
+/* The sample head and the hard gate of one decode step in one kernel (Alg. 1:
+ * the greedy step G_M and the sample rows' S_{T,theta} draw, then the probe
+ * token through the compatibility gate).  Same results as rgd_sample_head
+ * (without kept_mask) followed by
+ *   rgd_probe_gate(trie, rows / rows_per_group, rows_per_group, token_out, 1,
+ *                  rows_per_group, eos_token, max_len, state, row_active, ...):
+ * every active row draws its token first, and only then are the rows of a
+ * group masked by its gate outcome (the gate of group g runs once all
+ * rows_per_group rows of the group have their tokens).  Rows g*rows_per_group
+ * .. +rows_per_group-1 form group g; row g*rows_per_group is its probe (pass
+ * is_probe with those rows set, or temperature 0 there, for a greedy probe).
+ *   row_active   uint8 [rows] or NULL: read as by rgd_sample_head, then
+ *                updated in place by the gate
+ *   state        device rgd_gate_state [rows / rows_per_group], 4-byte
+ *                aligned; its `reserved` byte must be 0 between calls (the
+ *                kernel counts a group's finished rows there during the call
+ *                and leaves it at 0; rgd_gate_state_init sets it)
+ *   rows_per_group in [1, 255], dividing rows; max_len >= 1; trie non-NULL.
+ * One kernel on `stream`, launched as a programmatic dependent of the previous
+ * kernel on the stream (it is scheduled while that kernel finishes and waits
+ * for it before reading any input). */
+int rgd_sample_head_gated(int32_t rows, int32_t vocab, int32_t dtype, const void* logits,
+                          const uint8_t* is_probe, const float* temperature, const float* min_p,
+                          const uint64_t* seed, uint64_t step, uint8_t* row_active, int32_t* token_out,
+                          int32_t* kept_count, const rgd_trie* trie, int32_t rows_per_group,
+                          int32_t eos_token, int32_t max_len, rgd_gate_state* state, int32_t* dev_status,
+                          rgd_stream_t stream);
+
+/* One whole decode step of the gated loop: rgd_prefix_decode_attn over the
+ * step's rows, then rgd_sample_head_gated over the step's logits (two kernels
+ * on `stream`; the head's blocks are scheduled while the attention finishes).
+ * The logits are the caller's: the model between the attention output and the
+ * next-token logits (projections, MLP, LM head) is not part of this library.
+ * Arguments are those of the two calls, with rows = num_groups *
+ * rows_per_group and one row_active shared by both (the attention reads it,
+ * the gate updates it); out and lse receive the attention output.  The first
+ * error stops the step (nothing after it is launched). */
+int rgd_decode_step(const rgd_attn_shape* shape, const rgd_bf16* q, const rgd_bf16* k_pages,
+                    const rgd_bf16* v_pages, const int32_t* prompt_block_table, const int32_t* prompt_len,
+                    const int32_t* suffix_block_table, const int32_t* suffix_len, float softmax_scale,
+                    rgd_bf16* out, float* lse, void* workspace, size_t workspace_bytes, int32_t vocab,
+                    int32_t dtype, const void* logits, const uint8_t* is_probe, const float* temperature,
+                    const float* min_p, const uint64_t* seed, uint64_t step, uint8_t* row_active,
+                    int32_t* token_out, int32_t* kept_count, const rgd_trie* trie, int32_t eos_token,
+                    int32_t max_len, rgd_gate_state* state, int32_t* dev_status, rgd_stream_t stream);
 
 /* Soft compatibility gate (the appendix ablation's Alg. 2): one probe step per
  * group from the probe row's logits.  With y the greedy token (argmax, lowest

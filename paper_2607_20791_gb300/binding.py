@@ -51,12 +51,18 @@ _I32, _I64, _U64, _SZ, _F = ctypes.c_int32, ctypes.c_int64, ctypes.c_uint64, cty
 _SIGNATURES = {
     "rgd_last_error_string": (ctypes.c_char_p, []),
     "rgd_version": (ctypes.c_char_p, []),
+    "rgd_set_wait_limit_ns": (ctypes.c_int, [_U64]),
     "rgd_prefix_decode_attn_workspace_size": (_SZ, [ctypes.POINTER(AttnShape)]),
     "rgd_prefix_decode_attn": (ctypes.c_int, [ctypes.POINTER(AttnShape), _P, _P, _P, _P, _P, _P, _P, _P, _F,
                                                _P, _P, _P, _SZ, _P, _P]),
     "rgd_prefix_decode_attn_noalloc": (ctypes.c_int, [ctypes.POINTER(AttnShape), _P, _P, _P, _P, _P, _P, _P,
                                                        _P, _F, _P, _P, _P, _P]),
     "rgd_sample_head": (ctypes.c_int, [_I32, _I32, _I32, _P, _P, _P, _P, _P, _U64, _P, _P, _P, _P, _P, _P]),
+    "rgd_sample_head_gated": (ctypes.c_int, [_I32, _I32, _I32, _P, _P, _P, _P, _P, _U64, _P, _P, _P, _P, _I32,
+                                             _I32, _I32, _P, _P, _P]),
+    "rgd_decode_step": (ctypes.c_int, [ctypes.POINTER(AttnShape), _P, _P, _P, _P, _P, _P, _P, _F, _P, _P, _P,
+                                       _SZ, _I32, _I32, _P, _P, _P, _P, _P, _U64, _P, _P, _P, _P, _I32, _I32,
+                                       _P, _P, _P]),
     "rgd_trie_create": (ctypes.c_int, [_P, _P, _I32, _I32, ctypes.POINTER(_P)]),
     "rgd_trie_destroy": (ctypes.c_int, [_P]),
     "rgd_trie_info": (ctypes.c_int, [_P, ctypes.POINTER(_I32), ctypes.POINTER(_I32)]),
@@ -154,6 +160,11 @@ def rgd_version() -> str:
     return load_library().rgd_version().decode()
 
 
+def rgd_set_wait_limit_ns(limit_ns: int) -> None:
+    """Limit of the attention kernel's waits for later calls (0: the default, 2 s)."""
+    _check(load_library().rgd_set_wait_limit_ns(int(limit_ns)))
+
+
 def rgd_prefix_decode_attn_workspace_size(shape: AttnShape) -> int:
     n = load_library().rgd_prefix_decode_attn_workspace_size(ctypes.byref(shape))
     if n == 0:
@@ -227,6 +238,68 @@ def rgd_sample_head(logits, is_probe, temperature, min_p, seed, step: int, row_a
         _ptr(token_out, "token_out", torch.int32, numel=rows),
         _ptr(kept_count, "kept_count", torch.int32, optional=True, numel=rows),
         _ptr(kept_mask, "kept_mask", torch.uint8, optional=True, numel=rows * vocab),
+        _ptr(dev_status, "dev_status", torch.int32, optional=True, numel=1), _stream(stream)))
+
+
+def _logits_dtype(logits):
+    import torch
+    if logits.dim() != 2:
+        raise ValueError("logits must be [rows, vocab]")
+    dtype = {torch.float32: RGD_F32, torch.bfloat16: RGD_BF16}.get(logits.dtype)
+    if dtype is None:
+        raise TypeError("logits must be float32 or bfloat16")
+    return dtype
+
+
+def rgd_sample_head_gated(logits, is_probe, temperature, min_p, seed, step: int, row_active, token_out,
+                          kept_count, trie: "Trie", rows_per_group: int, eos_token: int, max_len: int, state,
+                          dev_status=None, stream=None) -> None:
+    """The sample head and the hard gate of one step in one kernel (see the C header)."""
+    import torch
+    dtype = _logits_dtype(logits)
+    rows, vocab = logits.shape
+    rpg = int(rows_per_group)
+    groups = rows // rpg if rpg > 0 else 0
+    _check(_call(load_library().rgd_sample_head_gated,
+        rows, vocab, dtype, _ptr(logits, "logits"),
+        _ptr(is_probe, "is_probe", torch.uint8, optional=True, numel=rows),
+        _ptr(temperature, "temperature", torch.float32, numel=rows), _ptr(min_p, "min_p", torch.float32, numel=rows),
+        _ptr(seed, "seed", (torch.int64, torch.uint64), numel=rows), int(step) & 0xFFFFFFFFFFFFFFFF,
+        _ptr(row_active, "row_active", torch.uint8, optional=True, numel=rows),
+        _ptr(token_out, "token_out", torch.int32, numel=rows),
+        _ptr(kept_count, "kept_count", torch.int32, optional=True, numel=rows),
+        trie.handle, rpg, int(eos_token), int(max_len), _state_ptr(state, groups),
+        _ptr(dev_status, "dev_status", torch.int32, optional=True, numel=1), _stream(stream)))
+
+
+def rgd_decode_step(shape: AttnShape, q, k_pages, v_pages, prompt_block_table, prompt_len, suffix_block_table,
+                    suffix_len, softmax_scale: float, out, lse, workspace, logits, is_probe, temperature, min_p,
+                    seed, step: int, row_active, token_out, kept_count, trie: "Trie", eos_token: int,
+                    max_len: int, state, dev_status=None, stream=None) -> None:
+    """One whole decode step: attention, then the gated sample head (see the C header)."""
+    import torch
+    n = _attn_sizes(shape)
+    dtype = _logits_dtype(logits)
+    rows, vocab = logits.shape
+    if rows != n["rows"]:
+        raise ValueError(f"logits has {rows} rows, the attention shape {n['rows']}")
+    ws_bytes = workspace.numel() * workspace.element_size() if isinstance(workspace, torch.Tensor) else 0
+    _check(_call(load_library().rgd_decode_step,
+        ctypes.byref(shape), _ptr(q, "q", torch.bfloat16, numel=n["q"]),
+        _ptr(k_pages, "k_pages", torch.bfloat16, numel=n["kv"]), _ptr(v_pages, "v_pages", torch.bfloat16, numel=n["kv"]),
+        _ptr(prompt_block_table, "prompt_block_table", torch.int32, numel=n["pbt"]),
+        _ptr(prompt_len, "prompt_len", torch.int32, numel=n["plen"]),
+        _ptr(suffix_block_table, "suffix_block_table", torch.int32, numel=n["sbt"]),
+        _ptr(suffix_len, "suffix_len", torch.int32, numel=n["rows"]), float(softmax_scale),
+        _ptr(out, "out", torch.bfloat16, numel=n["q"]), _ptr(lse, "lse", torch.float32, optional=True, numel=n["lse"]),
+        _ptr(workspace, "workspace"), ws_bytes, vocab, dtype, _ptr(logits, "logits"),
+        _ptr(is_probe, "is_probe", torch.uint8, optional=True, numel=rows),
+        _ptr(temperature, "temperature", torch.float32, numel=rows), _ptr(min_p, "min_p", torch.float32, numel=rows),
+        _ptr(seed, "seed", (torch.int64, torch.uint64), numel=rows), int(step) & 0xFFFFFFFFFFFFFFFF,
+        _ptr(row_active, "row_active", torch.uint8, optional=True, numel=rows),
+        _ptr(token_out, "token_out", torch.int32, numel=rows),
+        _ptr(kept_count, "kept_count", torch.int32, optional=True, numel=rows),
+        trie.handle, int(eos_token), int(max_len), _state_ptr(state, shape.num_groups),
         _ptr(dev_status, "dev_status", torch.int32, optional=True, numel=1), _stream(stream)))
 
 

@@ -57,6 +57,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <mutex>
 
@@ -126,6 +127,7 @@ struct AttnParams {
   int32_t G, rpg, Hq, Hkv, gq, num_pages, max_pp, max_sp;
   int32_t nq, nslots, C;
   float scale_log2;
+  uint64_t wait_ns;  // limit of every wait on another role or block (rgd_set_wait_limit_ns)
 };
 
 // Shared-memory carve-up (identical on host and device).  The ring is 1024-byte
@@ -270,7 +272,8 @@ __device__ __forceinline__ int64_t seq_page(const PieceIter& it, int64_t b, int6
 // Bounded wait that also gives up as soon as another role has given up.
 // A waiting thread sleeps inside try_wait (woken when the phase completes), so
 // warps parked on a barrier take no issue slots from the working ones.
-__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag) {
+__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag,
+                                              uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   if (*abort_flag) return false;
   const uint64_t t0 = globaltimer_ns();
@@ -278,7 +281,7 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
     if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
     if ((i & 63u) == 0) {
       if (*abort_flag) return false;
-      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      if (globaltimer_ns() - t0 > limit_ns) {
         *abort_flag = 1;
         return false;
       }
@@ -287,7 +290,8 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
 }
 
 // Bounded wait until *gen >= want (a shared counter another warp raises).
-__device__ __forceinline__ bool wait_slot_gen(int32_t* gen, int32_t want, volatile int32_t* abort_flag) {
+__device__ __forceinline__ bool wait_slot_gen(int32_t* gen, int32_t want, volatile int32_t* abort_flag,
+                                              uint64_t limit_ns) {
   volatile int32_t* g = gen;
   if (*g >= want) return true;
   const uint64_t t0 = globaltimer_ns();
@@ -295,7 +299,7 @@ __device__ __forceinline__ bool wait_slot_gen(int32_t* gen, int32_t want, volati
     if (*g >= want) return true;
     if ((i & 63u) == 0) {
       if (*abort_flag) return false;
-      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      if (globaltimer_ns() - t0 > limit_ns) {
         *abort_flag = 1;
         return false;
       }
@@ -542,8 +546,8 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
             const bool lead = in && (start || lane == 0);
             int stop = 0;
             if (lead && gq >= ns &&
-                (!wait_slot_gen(&s_slot_gen[gs], gq - ns, abort_flag) ||
-                 !wait_or_abort(&empty_bar[gs], (uint32_t)((gq / ns) - 1) & 1u, abort_flag)))
+                (!wait_slot_gen(&s_slot_gen[gs], gq - ns, abort_flag, p.wait_ns) ||
+                 !wait_or_abort(&empty_bar[gs], (uint32_t)((gq / ns) - 1) & 1u, abort_flag, p.wait_ns)))
               stop = 1;
             if (__any_sync(0xffffffffu, stop != 0)) {
               aborted = true;
@@ -572,6 +576,10 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
         gbase += __popc(starts);
       }
     }
+    // Every copy of this block is issued: a programmatic dependent of this
+    // kernel (the sample head) may be scheduled once every block has got here
+    // or exited.  It still waits for this kernel to complete before it reads.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   } else if (warp == kMmaWarp) {
     // ============================ QK issue ============================
     // One thread issues S = Q K^T for every group as soon as its pages have
@@ -588,19 +596,19 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
       Job cur = it.j0;
       int n_in = it.n0;
       for (bool more = b < e; ok && more; more = next_piece(p, gpre, it, pc, cur, n_in)) {
-        if (!wait_or_abort(&q_full, (uint32_t)pc & 1u, abort_flag)) break;
+        if (!wait_or_abort(&q_full, (uint32_t)pc & 1u, abort_flag, p.wait_ns)) break;
         tc_fence_after();
         const uint32_t qa = tmem + kQCol;
         for (int k0 = 0; k0 < n_in; k0 += kGroupPages) {
           const int ng = min(kGroupPages, n_in - k0);
           const int sb = gi % kSBufs;
           const int gs = gi % ns;
-          if (!wait_or_abort(&full_bar[gs], (uint32_t)(gi / ns) & 1u, abort_flag)) {
+          if (!wait_or_abort(&full_bar[gs], (uint32_t)(gi / ns) & 1u, abort_flag, p.wait_ns)) {
             ok = false;
             break;
           }
           // the S buffer is free once the softmax has read the group that used it last
-          if (gi >= kSBufs && !wait_or_abort(&s_empty[sb], (uint32_t)((gi / kSBufs) - 1) & 1u, abort_flag)) {
+          if (gi >= kSBufs && !wait_or_abort(&s_empty[sb], (uint32_t)((gi / kSBufs) - 1) & 1u, abort_flag, p.wait_ns)) {
             ok = false;
             break;
           }
@@ -637,12 +645,12 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
           const int ng = min(kGroupPages, n_in - k0);
           const int pb = gi % kPBufs;
           const int gs = gi % ns;
-          if (!wait_or_abort(&p_full[pb], (uint32_t)(gi / kPBufs) & 1u, abort_flag)) {
+          if (!wait_or_abort(&p_full[pb], (uint32_t)(gi / kPBufs) & 1u, abort_flag, p.wait_ns)) {
             ok = false;
             break;
           }
           // a piece's O buffer is free once the piece two back has been read out
-          if (k0 == 0 && pc >= 2 && !wait_or_abort(&o_free[pc & 1], (uint32_t)((pc >> 1) - 1) & 1u, abort_flag)) {
+          if (k0 == 0 && pc >= 2 && !wait_or_abort(&o_free[pc & 1], (uint32_t)((pc >> 1) - 1) & 1u, abort_flag, p.wait_ns)) {
             ok = false;
             break;
           }
@@ -706,7 +714,7 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
     constexpr int kChunks = D / 16;            // 16-column chunks of O (and 8-column chunks of Q)
     // warp-uniform bounded wait (TMEM loads and stores that follow are warp-collective)
     auto wwait = [&](uint64_t* bar, uint32_t parity, volatile int32_t* flag) {
-      return __all_sync(0xffffffffu, wait_or_abort(bar, parity, flag));
+      return __all_sync(0xffffffffu, wait_or_abort(bar, parity, flag, p.wait_ns));
     };
     // Q of job jb: this epilogue warp's share of its rows' query columns (8-column
     // chunks ei, ei + NE, ...), loaded first; then, if `after` is set, the wait for
@@ -1028,7 +1036,7 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
           __nanosleep(200);
           if ((i & 63u) == 0) {  // (warp-uniform exits: the loop holds warp collectives)
             if (__any_sync(0xffffffffu, *abort_flag != 0)) return false;
-            if (__any_sync(0xffffffffu, globaltimer_ns() - t0 > kWaitLimitNs)) {
+            if (__any_sync(0xffffffffu, globaltimer_ns() - t0 > p.wait_ns)) {
               *abort_flag = 1;
               return false;
             }
@@ -1042,7 +1050,7 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
         const uint64_t t0 = globaltimer_ns();
         while (tk == 0) {
           if (seen(__shfl_sync(0xffffffffu, lane == 0 ? ld_acquire_gpu(p.ticket + j) : 0, 0))) break;
-          if (__any_sync(0xffffffffu, globaltimer_ns() - t0 > kWaitLimitNs)) {
+          if (__any_sync(0xffffffffu, globaltimer_ns() - t0 > p.wait_ns)) {
             *abort_flag = 1;
             tk = -1;
             break;
@@ -1296,6 +1304,10 @@ int make_kv_map(CUtensorMap* map, const void* base, int64_t rows, int D, int box
   return RGD_OK;
 }
 
+// Limit of the kernel's waits on other roles and blocks, for the calls that
+// follow (rgd_set_wait_limit_ns).
+std::atomic<uint64_t> g_wait_ns{kWaitLimitNs};
+
 int device_sm_count() {
   int dev = 0, n = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 0;
@@ -1390,6 +1402,12 @@ size_t ws_total(const rgd_attn_shape* s) {
 
 using namespace rgd;
 
+extern "C" int rgd_set_wait_limit_ns(uint64_t limit_ns) {
+  clear_error();
+  g_wait_ns.store(limit_ns == 0 ? kWaitLimitNs : limit_ns, std::memory_order_relaxed);
+  return RGD_OK;
+}
+
 extern "C" size_t rgd_prefix_decode_attn_workspace_size(const rgd_attn_shape* shape) {
   clear_error();
   Plan pl;
@@ -1465,6 +1483,7 @@ extern "C" int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf1
   p.npref = pl.npref;
   p.C = pl.C;
   p.scale_log2 = softmax_scale * kLog2e;
+  p.wait_ns = g_wait_ns.load(std::memory_order_relaxed);
 
   cudaStream_t st = (cudaStream_t)stream;
   const int qpc = (pl.nq + 31) / 32;

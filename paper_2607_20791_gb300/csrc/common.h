@@ -31,6 +31,12 @@ int ensure_smem(Kernel k, int bytes, bool* done) {
   return RGD_OK;
 }
 
+// Argument checks of rgd_sample_head_gated (shared with rgd_decode_step, which
+// checks them before launching its first kernel).
+int check_gated_head(const char* fn, int32_t rows, int32_t vocab, int32_t dtype, const void* logits,
+                     const float* temperature, const float* min_p, const uint64_t* seed, const int32_t* token_out,
+                     const rgd_trie* trie, int32_t rows_per_group, int32_t max_len, const rgd_gate_state* state);
+
 }  // namespace rgd
 
 #define RGD_CHECK_ARG(cond, ...)                                        \

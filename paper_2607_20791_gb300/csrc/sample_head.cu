@@ -22,6 +22,7 @@
 
 #include "common.h"
 #include "ptx.cuh"
+#include "trie.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -49,7 +50,56 @@ struct HeadParams {
   int32_t* kept_count;
   uint8_t* kept_mask;
   int32_t* dev_status;
+  // the fused gate (gstate == nullptr: none): rows g * rpg .. g * rpg + rpg - 1
+  // form group g, whose probe token (row g * rpg) goes through the hard gate
+  TrieView trie;
+  rgd_gate_state* gstate;
+  uint8_t* gate_row_active;  // row_active, written by the gate
+  int32_t rpg, eos, max_len;
 };
+
+// The fused gate.  The thread that wrote a row's token counts the row as
+// finished in the top byte of its group's gate-state word {decision,
+// confirmed, done, reserved}; the group's last row to finish -- by then every
+// row of the group has drawn its token and read its activity flag -- feeds the
+// probe row's token to the hard gate (exactly rgd_probe_gate's step) and masks
+// the group's rows, and sets the count back to zero.  Nothing waits: a group
+// is gated by whichever of its rows ends last.
+__device__ __noinline__ void finish_row(const HeadParams& p, int row) {
+  const int g = row / p.rpg;
+  rgd_gate_state* st = p.gstate + g;
+  uint32_t* word = reinterpret_cast<uint32_t*>(&st->decision);
+  __threadfence();  // this row's token is visible before its count
+  const uint32_t old = atomicAdd(word, 1u << 24);
+  if ((int)(old >> 24) != p.rpg - 1) return;
+  __threadfence();  // the other rows counted themselves after writing their tokens
+  rgd_gate_state s;
+  s.node = st->node;
+  s.length = st->length;
+  s.steps = st->steps;
+  s.decisive_step = st->decisive_step;
+  s.decision = (uint8_t)(old & 0xffu);
+  s.confirmed = (uint8_t)((old >> 8) & 0xffu);
+  s.done = (uint8_t)((old >> 16) & 0xffu);
+  s.reserved = 0;
+  bool bad = false;
+  if (!s.done) {
+    const int32_t y = *reinterpret_cast<volatile const int32_t*>(p.token_out + (int64_t)g * p.rpg);
+    if (y < 0 && !(p.eos >= 0 && y == p.eos)) {
+      bad = true;  // (a probe row that was inactive or had bad parameters)
+    } else {
+      const bool root_has_children = __ldg(p.trie.child_begin + 1) > __ldg(p.trie.child_begin);
+      consume_token(p.trie, s, y, p.eos, p.max_len, root_has_children);
+    }
+  }
+  st->node = s.node;
+  st->length = s.length;
+  st->steps = s.steps;
+  st->decisive_step = s.decisive_step;
+  *word = (uint32_t)s.decision | ((uint32_t)s.confirmed << 8) | ((uint32_t)s.done << 16);  // count back to 0
+  if (bad && p.dev_status) atomicOr(p.dev_status, RGD_DEV_BAD_TOKEN);
+  mask_rows(s, p.gate_row_active, g, p.rpg);
+}
 
 // 16 bytes of logits: 4 fp32 or 8 bf16 elements.
 template <typename T>
@@ -179,11 +229,15 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
   const int rank = (int)cluster.block_rank();
   const int row = blockIdx.x / kClusterCtas;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  // launched as a programmatic dependent of the previous kernel on the stream:
+  // everything below may read what that kernel wrote
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 
   if (p.row_active && p.row_active[row] == 0) {  // uniform over the cluster
     if (rank == 0 && tid == 0) {
       p.token_out[row] = -1;
       if (p.kept_count) p.kept_count[row] = 0;
+      if (p.gstate) finish_row(p, row);
     }
     return;
   }
@@ -311,6 +365,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
         p.token_out[row] = A < p.vocab ? A : -1;
         if (p.kept_count) p.kept_count[row] = 1;
       }
+      if (p.gstate) finish_row(p, row);
     }
     return;
   }
@@ -487,6 +542,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
         }
         if (tok < 0) tok = lk;  // rounding put the target past the lane's last kept token
         p.token_out[row] = tok >= 0 ? tok : A;
+        if (p.gstate) finish_row(p, row);  // (one lane of one CTA of the cluster writes the token)
       }
     }
   }
@@ -497,40 +553,116 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
 
 using namespace rgd;
 
+namespace rgd {
+namespace {
+
+// The head kernel for the logits' type and alignment, launched as a
+// programmatic dependent of the previous kernel on the stream, so that its
+// blocks are scheduled while that kernel finishes (they wait for it before
+// reading anything).
+int launch_head(int32_t rows, int32_t vocab, int32_t dtype, const HeadParams& hp0, cudaStream_t st) {
+  const int es = dtype == RGD_F32 ? 4 : 2;
+  const int per_vec = 16 / es;
+  const int64_t stripe = 32 * per_vec;
+  const int64_t warps = (int64_t)kClusterCtas * kHeadWarps;
+  HeadParams hp = hp0;
+  hp.spw = (int32_t)((vocab + stripe * warps - 1) / (stripe * warps));
+  const bool aligned = ((int64_t)vocab * es) % 16 == 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(rows * kClusterCtas);
+  cfg.blockDim = dim3(kHeadThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e;
+  if (dtype == RGD_F32)
+    e = aligned ? cudaLaunchKernelEx(&cfg, sample_head_kernel<float, true>, hp)
+                : cudaLaunchKernelEx(&cfg, sample_head_kernel<float, false>, hp);
+  else
+    e = aligned ? cudaLaunchKernelEx(&cfg, sample_head_kernel<__nv_bfloat16, true>, hp)
+                : cudaLaunchKernelEx(&cfg, sample_head_kernel<__nv_bfloat16, false>, hp);
+  if (e == cudaSuccess) e = cudaGetLastError();
+  return e == cudaSuccess ? RGD_OK : cuda_error(e, "sample_head launch");
+}
+
+// Argument checks shared by both entry points.
+int check_head_args(const char* fn, int32_t rows, int32_t vocab, int32_t dtype, const void* logits,
+                    const float* temperature, const float* min_p, const uint64_t* seed, const int32_t* token_out) {
+  RGD_CHECK_ARG(rows >= 0, "%s: rows < 0", fn);
+  RGD_CHECK_ARG(vocab >= 1, "%s: vocab < 1", fn);
+  RGD_CHECK_ARG(dtype == RGD_F32 || dtype == RGD_BF16, "%s: dtype must be RGD_F32 or RGD_BF16", fn);
+  if (rows == 0) return RGD_OK;
+  RGD_CHECK_ARG(logits && temperature && min_p && seed && token_out,
+                "%s: logits/temperature/min_p/seed/token_out must be non-NULL", fn);
+  RGD_CHECK_ARG(aligned16(logits), "%s: logits must be 16-byte aligned", fn);
+  RGD_CHECK_ARG(rows <= 0x7fffffff / kClusterCtas, "%s: too many rows", fn);
+  const int es = dtype == RGD_F32 ? 4 : 2;
+  const int64_t stripe = 32 * (16 / es);
+  const int64_t warps = (int64_t)kClusterCtas * kHeadWarps;
+  if ((vocab + stripe * warps - 1) / (stripe * warps) > kMaxStripes)
+    return set_error(RGD_ERR_UNSUPPORTED, "%s: vocab %d too large (max %lld)", fn, vocab,
+                     (long long)(kMaxStripes * stripe * warps));
+  return RGD_OK;
+}
+
+}  // namespace
+}  // namespace rgd
+
 extern "C" int rgd_sample_head(int32_t rows, int32_t vocab, int32_t dtype, const void* logits,
                                const uint8_t* is_probe, const float* temperature, const float* min_p,
                                const uint64_t* seed, uint64_t step, const uint8_t* row_active,
                                int32_t* token_out, int32_t* kept_count, uint8_t* kept_mask,
                                int32_t* dev_status, rgd_stream_t stream) {
   clear_error();
-  RGD_CHECK_ARG(rows >= 0, "rgd_sample_head: rows < 0");
-  RGD_CHECK_ARG(vocab >= 1, "rgd_sample_head: vocab < 1");
-  RGD_CHECK_ARG(dtype == RGD_F32 || dtype == RGD_BF16, "rgd_sample_head: dtype must be RGD_F32 or RGD_BF16");
+  if (int rc = check_head_args("rgd_sample_head", rows, vocab, dtype, logits, temperature, min_p, seed, token_out))
+    return rc;
   if (rows == 0) return RGD_OK;
-  RGD_CHECK_ARG(logits && temperature && min_p && seed && token_out,
-                "rgd_sample_head: logits/temperature/min_p/seed/token_out must be non-NULL");
-  RGD_CHECK_ARG(aligned16(logits), "rgd_sample_head: logits must be 16-byte aligned");
-  RGD_CHECK_ARG(rows <= 0x7fffffff / kClusterCtas, "rgd_sample_head: too many rows");
-  const int es = dtype == RGD_F32 ? 4 : 2;
-  const int per_vec = 16 / es;
-  const int64_t stripe = 32 * per_vec;
-  const int64_t warps = (int64_t)kClusterCtas * kHeadWarps;
-  const int32_t spw = (int32_t)((vocab + stripe * warps - 1) / (stripe * warps));
-  if (spw > kMaxStripes)
-    return set_error(RGD_ERR_UNSUPPORTED, "rgd_sample_head: vocab %d too large (max %lld)", vocab,
-                     (long long)(kMaxStripes * stripe * warps));
-  const bool aligned = ((int64_t)vocab * es) % 16 == 0;
-  HeadParams hp{static_cast<const uint8_t*>(logits), rows, vocab, spw, is_probe, temperature, min_p, seed,
+  HeadParams hp{static_cast<const uint8_t*>(logits), rows, vocab, 0, is_probe, temperature, min_p, seed,
                 step, row_active, token_out, kept_count, kept_mask, dev_status};
-  const dim3 grid(rows * kClusterCtas), block(kHeadThreads);
-  cudaStream_t st = (cudaStream_t)stream;
-  if (dtype == RGD_F32) {
-    if (aligned) sample_head_kernel<float, true><<<grid, block, 0, st>>>(hp);
-    else sample_head_kernel<float, false><<<grid, block, 0, st>>>(hp);
-  } else {
-    if (aligned) sample_head_kernel<__nv_bfloat16, true><<<grid, block, 0, st>>>(hp);
-    else sample_head_kernel<__nv_bfloat16, false><<<grid, block, 0, st>>>(hp);
-  }
-  cudaError_t e = cudaGetLastError();
-  return e == cudaSuccess ? RGD_OK : cuda_error(e, "sample_head launch");
+  hp.gstate = nullptr;
+  return launch_head(rows, vocab, dtype, hp, (cudaStream_t)stream);
+}
+
+namespace rgd {
+
+int check_gated_head(const char* fn, int32_t rows, int32_t vocab, int32_t dtype, const void* logits,
+                     const float* temperature, const float* min_p, const uint64_t* seed, const int32_t* token_out,
+                     const rgd_trie* trie, int32_t rows_per_group, int32_t max_len, const rgd_gate_state* state) {
+  if (int rc = check_head_args(fn, rows, vocab, dtype, logits, temperature, min_p, seed, token_out)) return rc;
+  RGD_CHECK_ARG(trie != nullptr, "%s: trie is NULL", fn);
+  RGD_CHECK_ARG(rows_per_group >= 1 && rows_per_group <= 255, "%s: rows_per_group must be in [1, 255]", fn);
+  RGD_CHECK_ARG(rows % rows_per_group == 0, "%s: rows must be a multiple of rows_per_group", fn);
+  RGD_CHECK_ARG(max_len >= 1, "%s: max_len must be >= 1", fn);
+  if (rows == 0) return RGD_OK;
+  RGD_CHECK_ARG(state != nullptr, "%s: state is NULL", fn);
+  RGD_CHECK_ARG((reinterpret_cast<uintptr_t>(state) & 3u) == 0, "%s: state must be 4-byte aligned", fn);
+  return RGD_OK;
+}
+
+}  // namespace rgd
+
+extern "C" int rgd_sample_head_gated(int32_t rows, int32_t vocab, int32_t dtype, const void* logits,
+                                     const uint8_t* is_probe, const float* temperature, const float* min_p,
+                                     const uint64_t* seed, uint64_t step, uint8_t* row_active,
+                                     int32_t* token_out, int32_t* kept_count, const rgd_trie* trie,
+                                     int32_t rows_per_group, int32_t eos_token, int32_t max_len,
+                                     rgd_gate_state* state, int32_t* dev_status, rgd_stream_t stream) {
+  clear_error();
+  if (int rc = check_gated_head("rgd_sample_head_gated", rows, vocab, dtype, logits, temperature, min_p, seed,
+                                token_out, trie, rows_per_group, max_len, state))
+    return rc;
+  if (rows == 0) return RGD_OK;
+  HeadParams hp{static_cast<const uint8_t*>(logits), rows, vocab, 0, is_probe, temperature, min_p, seed,
+                step, row_active, token_out, kept_count, nullptr, dev_status};
+  hp.trie = TrieView{trie->child_begin, trie->child_tok, trie->child_node, trie->confirm};
+  hp.gstate = state;
+  hp.gate_row_active = row_active;
+  hp.rpg = rows_per_group;
+  hp.eos = eos_token;
+  hp.max_len = max_len;
+  return launch_head(rows, vocab, dtype, hp, (cudaStream_t)stream);
 }

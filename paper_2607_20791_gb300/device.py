@@ -12,7 +12,7 @@ from typing import Optional
 import numpy as np
 
 from . import binding
-from .workloads import AttnCase, HeadCase
+from .workloads import AttnCase, HeadCase, loop_spikes
 
 
 def _t(a: np.ndarray, device, dtype=None):
@@ -114,3 +114,69 @@ def head_to_device(case: HeadCase, device="cuda", with_mask: bool = False) -> De
         kept_count=torch.full((rows,), -7, dtype=torch.int32, device=device),
         kept_mask=(torch.zeros((rows, V), dtype=torch.uint8, device=device) if with_mask else None),
         dev_status=torch.zeros(1, dtype=torch.int32, device=device))
+
+
+class DeviceLoop:
+    """Device buffers and the captured CUDA graph of a whole gated loop
+    (:class:`workloads.LoopCase`): per step, the step's probe tokens are planted
+    in the logits, one rgd_decode_step runs (its tokens kept per step, its
+    attention output too when ``keep_history``), the logits go back to the
+    base, and every row active in the step grows its suffix by one token (the
+    KV of that token is already in the row's reserved pages).  A replay starts
+    from the prompt end: fresh gate states, every row active, empty suffixes."""
+
+    def __init__(self, case, stream, keep_history=True, kv=None):
+        import torch
+        self.case = case
+        a, h = case.attn, case.head
+        G, rpg, n = a.num_groups, a.rows_per_group, case.n_steps
+        R = G * rpg
+        self.att = attn_to_device(a, kv=kv)
+        self.head = head_to_device(h)
+        self.trie = binding.Trie(case.refusal_seqs, 2)
+        self.state = binding.new_gate_state(G)
+        self.row_active = torch.ones(R, dtype=torch.uint8, device="cuda")
+        self.snap = torch.empty_like(self.row_active)
+        self.suffix_len = torch.zeros(R, dtype=torch.int32, device="cuda")
+        idx, base = loop_spikes(case)
+        self.idx = torch.from_numpy(idx).cuda()
+        self.base = torch.from_numpy(base).cuda()
+        self.spike = torch.full((G,), case.spike, dtype=torch.float32, device="cuda")
+        self.flat = self.head.logits.view(-1)
+        self.tok = torch.full((n, R), -7, dtype=torch.int32, device="cuda")
+        self.out = (torch.zeros((n, R, a.num_q_heads, a.head_dim), dtype=torch.bfloat16, device="cuda")
+                    if keep_history else None)
+        self.status = torch.zeros(1, dtype=torch.int32, device="cuda")
+        self.stream = stream
+        self.graph = None
+
+    def _body(self):
+        s = self.stream.cuda_stream
+        a, c = self.att, self.case
+        binding.rgd_gate_state_init(self.state, a.shape.num_groups, stream=s)
+        self.row_active.fill_(1)
+        self.suffix_len.zero_()
+        for t in range(c.n_steps):
+            self.snap.copy_(self.row_active)
+            self.flat.scatter_(0, self.idx[t], self.spike)  # this step's probe tokens
+            out = self.out[t] if self.out is not None else a.out
+            binding.rgd_decode_step(a.shape, a.q, a.k_pages, a.v_pages, a.prompt_block_table, a.prompt_len,
+                                    a.suffix_block_table, self.suffix_len, a.softmax_scale, out, None,
+                                    a.workspace, self.head.logits, self.head.is_probe, self.head.temperature,
+                                    self.head.min_p, self.head.seed, t, self.row_active, self.tok[t], None,
+                                    self.trie, c.eos, c.max_len, self.state, self.status, stream=s)
+            self.flat.scatter_(0, self.idx[t], self.base[t])  # back to the base logits
+            self.suffix_len.add_(self.snap)  # every row active this step appended its token
+
+    def capture(self):
+        import torch
+        with torch.cuda.stream(self.stream):
+            self._body()  # eager run first (kernel attributes are set outside capture)
+            torch.cuda.synchronize()
+            self.graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(self.graph, stream=self.stream):
+                self._body()
+        torch.cuda.synchronize()
+
+    def close(self):
+        self.trie.close()

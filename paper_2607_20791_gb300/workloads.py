@@ -77,20 +77,22 @@ def make_attn_case(name: str, num_groups: int, rows_per_group: int, num_q_heads:
                    num_kv_heads: int, head_dim: int, prompt_lens: Sequence[int],
                    suffix_lens: Sequence[int], seed: int,
                    row_active: Optional[np.ndarray] = None, spare_pages: int = 3,
-                   with_kv: bool = True, min_table_cols: int = 1) -> AttnCase:
+                   with_kv: bool = True, min_table_cols: int = 1, suffix_room: int = 0) -> AttnCase:
     """Draw Q and paged K/V ~ N(0,1) in bf16 with pages shuffled in the pool.
 
     Pages of all prompts and suffixes are assigned through a seeded random
     permutation of the pool, so consecutive logical pages are scattered the way
     a paged KV cache is after some serving time.  Unused block-table entries
-    hold -1.
+    hold -1.  ``suffix_room`` extra tokens of pages are assigned to every row's
+    suffix (filled like the rest), so that a decode loop can grow the suffixes
+    by that many tokens without a new page.
     """
     G, rpg = int(num_groups), int(rows_per_group)
     R = G * rpg
     prompt_lens = np.asarray(prompt_lens, dtype=np.int32).reshape(G)
     suffix_lens = np.asarray(suffix_lens, dtype=np.int32).reshape(R)
     ppages = (prompt_lens + PAGE_SIZE - 1) // PAGE_SIZE
-    spages = (suffix_lens + PAGE_SIZE - 1) // PAGE_SIZE
+    spages = (suffix_lens + int(suffix_room) + PAGE_SIZE - 1) // PAGE_SIZE
     total = int(ppages.sum() + spages.sum())
     num_pages = total + int(spare_pages)
     rng = _rng(seed, 1)
@@ -270,6 +272,36 @@ def make_probe_streams(refusal_seqs: Sequence[np.ndarray], groups: int, n_steps:
     return out
 
 
+def loop_probe_streams(refusal_seqs: Sequence[np.ndarray], groups: int, n_steps: int, vocab: int,
+                       seed: int, eos: int) -> np.ndarray:
+    """Greedy probe streams [groups, n_steps] for a whole gated loop, one kind per
+    group in turn: (0) a refusal sequence in full, then random tokens to the
+    cap; (1) a refusal sequence in full, then random tokens, then the stop token
+    at a random later step; (2) part of a sequence, then a diverging token;
+    (3) random from the start; (4) a proper prefix of a sequence, then the stop
+    token.  Random tokens never equal the stop token."""
+    rng = _rng(seed, 9)
+    out = rng.integers(0, vocab, size=(groups, n_steps)).astype(np.int32)
+    out[out == eos] = (eos + 1) % vocab
+    for g in range(groups):
+        kind = g % 5
+        if kind == 3 or not refusal_seqs:
+            continue
+        s = refusal_seqs[int(rng.integers(len(refusal_seqs)))]
+        if kind in (0, 1):
+            k = min(len(s), n_steps)
+            out[g, :k] = s[:k]
+            if kind == 1 and k + 1 < n_steps:
+                out[g, int(rng.integers(k, n_steps))] = eos
+        else:
+            k = int(rng.integers(1, len(s))) if len(s) > 1 else 0
+            k = min(k, n_steps - 1)
+            out[g, :k] = s[:k]
+            if kind == 4:
+                out[g, k] = eos
+    return out
+
+
 # --------------------------------------------------------------------------
 # the five workloads
 # --------------------------------------------------------------------------
@@ -380,6 +412,69 @@ def high_batch(seed: int = 0, with_kv: bool = True, lognormal_sigma: float = 1.0
                           row_active=active)
     gate = _gate_for_step("high_batch", seed, G, rpg, V, 64, 2, 8, 128)
     return StepCase("high_batch", attn, head, gate)
+
+
+@dataclasses.dataclass
+class LoopCase:
+    """A whole gated decode loop (Alg. 1 with the probe and the sample rows of
+    each prompt decoding side by side): every row starts at the end of its
+    prompt (empty suffix) and appends one token per step it is active, in the
+    suffix pages reserved for it; each step's logits are ``head.logits`` with
+    the probe row of group g raised to ``spike`` at ``probe_streams[g, step]``,
+    so that the greedy probe follows a planted stream."""
+
+    name: str
+    attn: AttnCase
+    head: HeadCase
+    refusal_seqs: List[np.ndarray]
+    probe_streams: np.ndarray   # int32 [G, n_steps]
+    eos: int
+    max_len: int                # L, the probe's length cap
+    gate_cap: int               # c of Alg. 1 (does not change the hard gate's outcome)
+    n_steps: int
+    spike: float = 64.0
+
+
+def llama8b_loop(seed: int = 0, n_steps: int = 128, with_kv: bool = True) -> LoopCase:
+    """The Llama-3-8B-shaped step as a loop of ``n_steps`` decode steps from the
+    prompt end: 16 prompts of U[512, 2048] tokens, 1 probe + 4 sample rows each,
+    32 q / 8 kv heads, head dim 128; fp32 Zipf logits over 128256 with the
+    config's temperatures and min-p; 64 refusal sequences of length 2-8; the
+    probe cap L = 128 and the gate cap c = 3 (App. D); the stop token is the
+    last vocabulary entry; the probes follow :func:`loop_probe_streams`."""
+    G, rpg, V = 16, 5, 128256
+    eos = V - 1
+    rng = _rng(seed, 24)
+    plens = rng.integers(512, 2049, size=G)
+    attn = make_attn_case("llama8b_loop", G, rpg, 32, 8, 128, plens, np.zeros(G * rpg, np.int32), seed,
+                          with_kv=with_kv, suffix_room=n_steps)
+    logits = zipf_logits(G * rpg, V, seed)
+    is_probe = np.tile([1, 0, 0, 0, 0], G)
+    temps = np.tile([0.0, 1.0, 1.5, 2.0, 3.0], G)
+    minp = np.repeat([0.05 if g % 2 == 0 else 0.1 for g in range(G)], rpg)
+    head = make_head_case("llama8b_loop", logits, "f32", is_probe, temps, minp, seed)
+    seqs = make_refusal_set(64, 2, 8, V, seed, avoid=[eos])
+    streams = loop_probe_streams(seqs, G, n_steps, V, seed, eos)
+    return LoopCase(name="llama8b_loop", attn=attn, head=head, refusal_seqs=seqs, probe_streams=streams,
+                    eos=eos, max_len=128, gate_cap=3, n_steps=n_steps)
+
+
+def loop_spikes(case: LoopCase):
+    """Flat logit indices [n_steps, G] of each step's planted probe tokens and
+    the base values they hold outside that step (float32 [n_steps, G])."""
+    G, rpg, V = case.attn.num_groups, case.attn.rows_per_group, case.head.vocab
+    rows = np.arange(G, dtype=np.int64) * rpg
+    idx = rows[None, :] * V + case.probe_streams.T.astype(np.int64)
+    base = case.head.logits.reshape(-1)[idx].astype(np.float32)
+    return idx, base
+
+
+def loop_step_logits(case: LoopCase, step: int) -> np.ndarray:
+    """The logits of one loop step (a copy of the base with the step's spikes)."""
+    out = case.head.logits.copy()
+    rpg = case.attn.rows_per_group
+    out[np.arange(case.attn.num_groups) * rpg, case.probe_streams[:, step]] = case.spike
+    return out
 
 
 SWEEP_BATCHES = (1, 8, 64, 256, 1024)

@@ -61,6 +61,30 @@ def test_version_and_argument_errors_without_gpu(lib_path):
     assert rc == binding.RGD_ERR_INVALID_ARG and b"top_k" in lib.rgd_last_error_string()
 
 
+def test_gated_head_and_decode_step_argument_errors_without_gpu(lib_path):
+    """The fused head + gate and the one-call step refuse bad arguments on the
+    host, before any launch (the trie handle is not looked at before that)."""
+    lib = binding.load_library(lib_path)
+    P = 16  # any non-NULL, 16-byte aligned stand-in pointer
+    args = lambda rows, rpg, max_len, trie=1, state=P: (rows, 100, 0, P, None, P, P, P, 0, None, P, None, trie,
+                                                       rpg, -1, max_len, state, None, None)
+    assert lib.rgd_sample_head_gated(*args(6, 4, 8)) == binding.RGD_ERR_INVALID_ARG  # 6 rows, groups of 4
+    assert b"multiple" in lib.rgd_last_error_string()
+    assert lib.rgd_sample_head_gated(*args(6, 3, 0)) == binding.RGD_ERR_INVALID_ARG  # max_len 0
+    assert lib.rgd_sample_head_gated(*args(6, 3, 8, trie=None)) == binding.RGD_ERR_INVALID_ARG
+    assert lib.rgd_sample_head_gated(*args(6, 256, 8)) == binding.RGD_ERR_INVALID_ARG  # rows_per_group > 255
+    assert lib.rgd_sample_head_gated(*args(6, 3, 8, state=None)) == binding.RGD_ERR_INVALID_ARG
+    assert lib.rgd_sample_head_gated(*args(6, 3, 8, state=P + 2)) == binding.RGD_ERR_INVALID_ARG  # misaligned
+    assert lib.rgd_sample_head_gated(*args(0, 3, 8)) == 0  # an empty batch launches nothing
+    shape = binding.AttnShape(num_groups=2, rows_per_group=3, num_q_heads=4, num_kv_heads=1, head_dim=128,
+                              page_size=16, num_pages=4, max_prompt_pages=1, max_suffix_pages=1, num_ctas=4)
+    # the head's arguments are checked first: max_len 0 is refused before the attention's
+    rc = lib.rgd_decode_step(ctypes.byref(shape), P, P, P, P, P, P, P, 0.1, P, None, P, 1 << 20, 100, 0, P, None,
+                             P, P, P, 0, None, P, None, 1, -1, 0, P, None, None)
+    assert rc == binding.RGD_ERR_INVALID_ARG and b"max_len" in lib.rgd_last_error_string()
+    assert lib.rgd_set_wait_limit_ns(0) == 0
+
+
 def test_workspace_size_grows_with_blocks(lib_path):
     lib = binding.load_library(lib_path)
     s = binding.AttnShape(num_groups=16, rows_per_group=5, num_q_heads=32, num_kv_heads=8, head_dim=128,
