@@ -34,6 +34,8 @@ constexpr int kHeadThreads = 256;
 constexpr int kHeadWarps = kHeadThreads / 32;
 constexpr int kBatch = 4;        // 16-byte loads in flight per lane
 constexpr int kMaxStripes = 64;  // stripes per warp whose sums are kept for the draw
+constexpr int kSparseStripes = 16;  // stripes per warp for which lane maxima are kept
+constexpr int kSparseHits = 16;     // vectors one lane re-reads at most in the sparse pass 2
 
 struct HeadParams {
   const uint8_t* logits;
@@ -58,46 +60,51 @@ struct HeadParams {
   int32_t rpg, eos, max_len;
 };
 
-// The fused gate.  The thread that wrote a row's token counts the row as
-// finished in the top byte of its group's gate-state word {decision,
-// confirmed, done, reserved}; the group's last row to finish -- by then every
-// row of the group has drawn its token and read its activity flag -- feeds the
-// probe row's token to the hard gate (exactly rgd_probe_gate's step) and masks
-// the group's rows, and sets the count back to zero.  Nothing waits: a group
-// is gated by whichever of its rows ends last.
-__device__ __noinline__ void finish_row(const HeadParams& p, int row) {
+// The fused gate.  The thread that writes a row's token then counts the row as
+// finished in the top byte of its group's gate-state word {decision, confirmed,
+// done, reserved}.  The probe row's thread first feeds its token to the hard
+// gate (exactly rgd_probe_gate's step): it writes the state's integer fields
+// directly and the decision, confirmed and done bytes by atomics, which leave
+// the count in the top byte alone.  The group's last row to finish -- by then
+// every row of the group has drawn its token and read its activity flag, and
+// the probe's outcome is in the word its count returns -- masks the group's rows
+// and sets the count back to zero.  Nothing waits, and the trie walk runs on
+// the probe row, whose greedy path ends long before the sampled rows'.
+__device__ __noinline__ void finish_row(const HeadParams& p, int row, int32_t tok) {
   const int g = row / p.rpg;
   rgd_gate_state* st = p.gstate + g;
   uint32_t* word = reinterpret_cast<uint32_t*>(&st->decision);
-  __threadfence();  // this row's token is visible before its count
-  const uint32_t old = atomicAdd(word, 1u << 24);
-  if ((int)(old >> 24) != p.rpg - 1) return;
-  __threadfence();  // the other rows counted themselves after writing their tokens
-  rgd_gate_state s;
-  s.node = st->node;
-  s.length = st->length;
-  s.steps = st->steps;
-  s.decisive_step = st->decisive_step;
-  s.decision = (uint8_t)(old & 0xffu);
-  s.confirmed = (uint8_t)((old >> 8) & 0xffu);
-  s.done = (uint8_t)((old >> 16) & 0xffu);
-  s.reserved = 0;
-  bool bad = false;
-  if (!s.done) {
-    const int32_t y = *reinterpret_cast<volatile const int32_t*>(p.token_out + (int64_t)g * p.rpg);
-    if (y < 0 && !(p.eos >= 0 && y == p.eos)) {
-      bad = true;  // (a probe row that was inactive or had bad parameters)
-    } else {
-      const bool root_has_children = __ldg(p.trie.child_begin + 1) > __ldg(p.trie.child_begin);
-      consume_token(p.trie, s, y, p.eos, p.max_len, root_has_children);
+  if (row == g * p.rpg) {
+    const uint32_t w0 = *reinterpret_cast<volatile uint32_t*>(word);  // (only this thread changes the low bytes)
+    rgd_gate_state s;
+    s.done = (uint8_t)((w0 >> 16) & 0xffu);
+    if (!s.done) {
+      if (tok < 0 && !(p.eos >= 0 && tok == p.eos)) {
+        if (p.dev_status) atomicOr(p.dev_status, RGD_DEV_BAD_TOKEN);  // (an inactive or rejected probe row)
+      } else {
+        s.node = st->node;
+        s.length = st->length;
+        s.steps = st->steps;
+        s.decisive_step = st->decisive_step;
+        s.decision = (uint8_t)(w0 & 0xffu);
+        s.confirmed = (uint8_t)((w0 >> 8) & 0xffu);
+        const bool root_has_children = __ldg(p.trie.child_begin + 1) > __ldg(p.trie.child_begin);
+        consume_token(p.trie, s, tok, p.eos, p.max_len, root_has_children);
+        st->node = s.node;
+        st->length = s.length;
+        st->steps = s.steps;
+        st->decisive_step = s.decisive_step;
+        atomicAnd(word, 0xff000000u);
+        atomicOr(word, (uint32_t)s.decision | ((uint32_t)s.confirmed << 8) | ((uint32_t)s.done << 16));
+      }
     }
   }
-  st->node = s.node;
-  st->length = s.length;
-  st->steps = s.steps;
-  st->decisive_step = s.decisive_step;
-  *word = (uint32_t)s.decision | ((uint32_t)s.confirmed << 8) | ((uint32_t)s.done << 16);  // count back to 0
-  if (bad && p.dev_status) atomicOr(p.dev_status, RGD_DEV_BAD_TOKEN);
+  const uint32_t old = atomicAdd(word, 1u << 24);
+  if ((int)(old >> 24) != p.rpg - 1) return;
+  *word = old & 0x00ffffffu;  // the count back to 0 (every row of the group has counted itself)
+  rgd_gate_state s;
+  s.decision = (uint8_t)(old & 0xffu);
+  s.done = (uint8_t)((old >> 16) & 0xffu);
   mask_rows(s, p.gate_row_active, g, p.rpg);
 }
 
@@ -182,6 +189,9 @@ struct Shared {
   int32_t red_c[kHeadWarps];
   float stripe_sum[kHeadWarps][kMaxStripes];
   float stripe_max[kHeadWarps][kMaxStripes];
+  // pass 1: each lane's maximum over its vector of each stripe (spw <=
+  // kSparseStripes); pass 2 overwrites a lane's column with its partial sums
+  float lane_part[kHeadWarps][kSparseStripes][33];
   uint8_t stripe_list[kHeadWarps][kMaxStripes];  // pass 2: the stripes a warp re-reads
   // pushed by every CTA of the cluster into every CTA's copy (slot = rank)
   float cta_max[kClusterCtas];
@@ -237,7 +247,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
     if (rank == 0 && tid == 0) {
       p.token_out[row] = -1;
       if (p.kept_count) p.kept_count[row] = 0;
-      if (p.gstate) finish_row(p, row);
+      if (p.gstate) finish_row(p, row, -1);
     }
     return;
   }
@@ -287,7 +297,9 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
           bi = base + k;
         }
       }
-      // the stripe's maximum: pass 2 skips stripes that cannot hold a kept token
+      // the lane's and the stripe's maxima: pass 2 skips vectors and stripes
+      // that cannot hold a kept token
+      if (s0 + b < kSparseStripes) sh.lane_part[warp][s0 + b][lane] = sm;
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) sm = fmaxf(sm, __shfl_xor_sync(0xffffffffu, sm, o));
       if (lane == 0) sh.stripe_max[warp][s0 + b] = sm;
@@ -357,15 +369,16 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
                    A >= p.vocab;
   if (greedy || bad) {
     if (rank == 0 && tid == 0) {
+      int32_t tok = -1;
       if (bad && !greedy) {
         if (p.dev_status) atomicOr(p.dev_status, RGD_DEV_BAD_PARAM);
-        p.token_out[row] = -1;
         if (p.kept_count) p.kept_count[row] = 0;
       } else {
-        p.token_out[row] = A < p.vocab ? A : -1;
+        tok = A < p.vocab ? A : -1;
         if (p.kept_count) p.kept_count[row] = 1;
       }
-      if (p.gstate) finish_row(p, row);
+      p.token_out[row] = tok;
+      if (p.gstate) finish_row(p, row, tok);  // (this row is done: no further counting below)
     }
     return;
   }
@@ -376,12 +389,69 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
   uint8_t* mask = p.kept_mask ? p.kept_mask + (int64_t)row * p.vocab : nullptr;
   KSum wsum;  // identical in every lane
   int32_t cnt = 0;
-  // Only stripes whose maximum reaches the cutoff can hold a kept token: the
-  // warp lists them (in index order) and re-reads just those; the others' sums
-  // are 0.  With a kept mask requested every stripe is visited.
   for (int st = lane; st < spw; st += 32) sh.stripe_sum[warp][st] = 0.f;
+  // Sparse form: a lane's maxima from pass 1 say which of its vectors can hold
+  // a kept token.  Every lane re-reads only its own such vectors (one trip to
+  // L2 per four of them, instead of one per four stripes any lane hits), writes
+  // each one's kept weight sum in its column of lane_part, and the warp sums
+  // every stripe some lane hit.
+  uint32_t hits = 0;
+  bool sparse = mask == nullptr && spw <= kSparseStripes;
+  if (sparse) {
+    for (int st = 0; st < spw; ++st) hits |= sh.lane_part[warp][st][lane] >= cut ? (1u << st) : 0u;
+    sparse = __all_sync(0xffffffffu, __popc(hits) <= kSparseHits);
+  }
+  if (sparse) {
+    for (int st = 0; st < spw; ++st) sh.lane_part[warp][st][lane] = 0.f;
+    uint32_t hm = hits;
+    while (hm) {  // (lanes differ in their trip counts; no warp-wide operation inside)
+      uint4 w[kBatch];
+      int sidx[kBatch];
+#pragma unroll
+      for (int b = 0; b < kBatch; ++b) {
+        sidx[b] = -1;
+        if (hm) {
+          sidx[b] = __ffs(hm) - 1;
+          hm &= hm - 1;
+          w[b] = load_vec<T, kAligned>(rowp, elem(warp, sidx[b], 0), p.vocab, drop_pol);
+        }
+      }
+#pragma unroll
+      for (int b = 0; b < kBatch; ++b) {
+        if (sidx[b] < 0) break;
+        const int32_t base = (int32_t)elem(warp, sidx[b], 0);
+        uint32_t km = 0;
+#pragma unroll
+        for (int k = 0; k < kN; ++k) km |= (V::get(w[b], k) >= cut && base + k < p.vocab) ? (1u << k) : 0u;
+        cnt += __popc(km);
+        float ls = 0.f;
+        while (km) {
+          const int k = __ffs(km) - 1;
+          km &= km - 1;
+          ls += ex2_approx(__fsub_rn(V::get(w[b], k), M) * kexp);
+        }
+        sh.lane_part[warp][sidx[b]][lane] = ls;
+      }
+    }
+    __syncwarp();
+    // the sums of the stripes where some lane re-read a vector (the others stay 0),
+    // each by a butterfly over the lanes (the same value in every lane), in stripe order
+    uint32_t any = __reduce_or_sync(0xffffffffu, hits);
+    while (any) {
+      const int st = __ffs(any) - 1;
+      any &= any - 1;
+      float S = sh.lane_part[warp][st][lane];
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) S += __shfl_xor_sync(0xffffffffu, S, o);
+      if (lane == 0) sh.stripe_sum[warp][st] = S;
+      wsum.add(S);
+    }
+  }
+  // Dense form: only stripes whose maximum reaches the cutoff can hold a kept
+  // token: the warp lists them (in index order) and re-reads just those; the
+  // others' sums are 0.  With a kept mask requested every stripe is visited.
   int nlist = 0;
-  for (int s0 = 0; s0 < spw; s0 += 32) {
+  for (int s0 = 0; s0 < spw && !sparse; s0 += 32) {
     const bool hit = s0 + lane < spw && (mask != nullptr || sh.stripe_max[warp][s0 + lane] >= cut);
     const uint32_t bal = __ballot_sync(0xffffffffu, hit);
     if (hit) sh.stripe_list[warp][nlist + __popc(bal & ((1u << lane) - 1u))] = (uint8_t)(s0 + lane);
@@ -446,6 +516,9 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
     }
   }
   cluster.sync();  // #2: every CTA's sums are in every CTA's shared memory
+  // a sampled row other than the probe is counted by an idle warp, off the
+  // draw's path (every CTA of the cluster read its activity flag long ago)
+  if (p.gstate && rank == kClusterCtas - 1 && tid == 32 && row % p.rpg != 0) finish_row(p, row, -1);
 
   // ---- the draw: target u * Z; CTA, warp and stripe by prefix sums in index
   // order; then the stripe's lanes and the lane's elements --------------------
@@ -541,8 +614,11 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
           }
         }
         if (tok < 0) tok = lk;  // rounding put the target past the lane's last kept token
-        p.token_out[row] = tok >= 0 ? tok : A;
-        if (p.gstate) finish_row(p, row);  // (one lane of one CTA of the cluster writes the token)
+        if (tok < 0) tok = A;
+        p.token_out[row] = tok;
+        // (one lane of one CTA of the cluster writes the token; a sampled probe
+        // row's token goes through the gate here)
+        if (p.gstate && row % p.rpg == 0) finish_row(p, row, tok);
       }
     }
   }
