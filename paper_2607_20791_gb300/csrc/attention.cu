@@ -1118,12 +1118,84 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
         }
       }
       const float inv = Lt > 0.f ? 1.f / Lt : 0.f;
-      // O in 16-column chunks: epilogue warp ei of a quarter takes chunks ei,
-      // ei + NE, ...; copies >= 1 pass theirs to copy 0 through shared memory
+      // The block's last piece, with copies: the ring is idle (every group's
+      // PV is done), so it holds all the copies' O at once -- each epilogue
+      // warp writes its copy's columns there, one barrier, and the R warps of a
+      // row block then each sum the copies over their own D/R columns and
+      // write those (instead of one barrier per 16 columns and copy 0's warp
+      // writing every column).
+      const bool whole = R > 1 && !more;
+      if (whole) {
+        float* stg = reinterpret_cast<float*>(smem);  // [R * qpc][D][32]
+        float* mine = stg + (size_t)(cp * qpc + rb) * D * 32;
+        if (out_ok) {
+#pragma unroll 1
+          for (int col = 0; col < D; col += 32) {
+            uint32_t r0[16], r1[16];
+            tmem_ld16(tl + ocol + col, r0);
+            tmem_ld16(tl + ocol + col + 16, r1);
+            tmem_ld_wait();
+#pragma unroll
+            for (int t = 0; t < 16; ++t) {
+              mine[(col + t) * 32 + lane] = __uint_as_float(r0[t]) * wself;
+              mine[(col + 16 + t) * 32 + lane] = __uint_as_float(r1[t]) * wself;
+            }
+          }
+        }
+        epi_sync();
+        constexpr int kCols = D / R;  // this warp's output columns (a multiple of 16)
+        const bool row_ok = out_ok && r < nq;
+        const bool out_row = row_ok && ((rowbits[rr >> 5] >> (rr & 31)) & 1u);
+#pragma unroll 1
+        for (int c0 = 0; c0 < kCols; c0 += 16) {
+          const int col = cp * kCols + c0;
+          if (!row_ok) break;
+          float o[16];
+#pragma unroll
+          for (int t = 0; t < 16; ++t) o[t] = 0.f;
+          for (int c2 = 0; c2 < R; ++c2) {
+            const float* src = stg + ((size_t)(c2 * qpc + rb) * D + col) * 32 + lane;
+#pragma unroll
+            for (int t = 0; t < 16; ++t) o[t] += src[t * 32];
+          }
+          if (!split || fused) {
+            if (!out_row) continue;
+            if (fused) {
+#pragma unroll
+              for (int t = 0; t < 16; ++t) o[t] *= a;
+#pragma unroll
+              for (int k = 0; k < 2; ++k) {
+                if (k >= nparts) break;
+                const float4* src4 = reinterpret_cast<const float4*>(pref_o + (k * nq + r) * (D + 4) + col);
+#pragma unroll
+                for (int t = 0; t < 4; ++t) {
+                  const float4 v = src4[t];
+                  o[4 * t] += bk[k] * v.x;
+                  o[4 * t + 1] += bk[k] * v.y;
+                  o[4 * t + 2] += bk[k] * v.z;
+                  o[4 * t + 3] += bk[k] * v.w;
+                }
+              }
+            }
+            uint4* dst = reinterpret_cast<uint4*>(p.out + ((int64_t)rr * p.Hq + hq) * D + col);
+            dst[0] = make_uint4(pack_bf16x2(o[0] * inv, o[1] * inv), pack_bf16x2(o[2] * inv, o[3] * inv),
+                                pack_bf16x2(o[4] * inv, o[5] * inv), pack_bf16x2(o[6] * inv, o[7] * inv));
+            dst[1] = make_uint4(pack_bf16x2(o[8] * inv, o[9] * inv), pack_bf16x2(o[10] * inv, o[11] * inv),
+                                pack_bf16x2(o[12] * inv, o[13] * inv), pack_bf16x2(o[14] * inv, o[15] * inv));
+          } else {
+            float4* dst = reinterpret_cast<float4*>(p.slot_o + (s_idx * nq + r) * D + col);
+#pragma unroll
+            for (int t = 0; t < 4; ++t) dst[t] = make_float4(o[4 * t], o[4 * t + 1], o[4 * t + 2], o[4 * t + 3]);
+          }
+        }
+      }
+      // Otherwise O in 16-column chunks: epilogue warp ei of a quarter takes
+      // chunks ei, ei + NE, ...; copies >= 1 pass theirs to copy 0 through
+      // shared memory
       constexpr int rounds = (kChunks + NE - 1) / NE;
       const int my_stage = ((cp - 1) * qpc + rb) * NE + ei;  // (for copies >= 1)
 #pragma unroll 1
-      for (int rd = 0; rd < rounds; ++rd) {
+      for (int rd = 0; rd < (whole ? 0 : rounds); ++rd) {
         const int ch = ei + rd * NE;
         const bool has = ch < kChunks && out_ok;
         const int col = ch * 16;
