@@ -272,9 +272,8 @@ __device__ __forceinline__ int64_t seq_page(const PieceIter& it, int64_t b, int6
 // Bounded wait that also gives up as soon as another role has given up.
 // A waiting thread sleeps inside try_wait (woken when the phase completes), so
 // warps parked on a barrier take no issue slots from the working ones.
-__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag,
-                                              uint64_t limit_ns) {
-  if (mbar_try_wait(bar, parity)) return true;
+__device__ __noinline__ bool wait_or_abort_slow(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag,
+                                                uint64_t limit_ns) {
   if (*abort_flag) return false;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {
@@ -287,6 +286,13 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
       }
     }
   }
+}
+// (the loop is out of line: it is only reached when the phase has not completed
+// at the first look, and one copy keeps the kernels' code small)
+__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int32_t* abort_flag,
+                                              uint64_t limit_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  return wait_or_abort_slow(bar, parity, abort_flag, limit_ns);
 }
 
 // Bounded wait until *gen >= want (a shared counter another warp raises).
@@ -1342,6 +1348,14 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
   if (warp == kMmaWarp) tmem_dealloc(tmem, kTmemCols);
 }
 
+}  // namespace
+}  // namespace rgd
+
+#include "attention_t.cuh"
+
+namespace rgd {
+namespace {
+
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
@@ -1389,7 +1403,8 @@ int device_sm_count() {
 
 struct Plan {
   int nq, nslots, C, J, npref;
-  SmemLayout smem;
+  bool transposed;  // attn_t_kernel (nq <= 32) rather than attn_tc_kernel
+  int smem_bytes;   // dynamic shared memory of the launch
   size_t ticket_off, ml_off, o_off, total;
 };
 
@@ -1433,11 +1448,27 @@ int make_plan(const rgd_attn_shape* s, Plan* pl) {
   // to four slots; one staged partial is the minimum (the merges go through
   // that area).
   const int rows = s->num_groups * s->rows_per_group;
+  pl->transposed = pl->nq <= kTN;
+  pl->nslots = 0;
+  pl->npref = 0;
+  if (pl->transposed) {
+    // as many 8-page group slots as fit (three at head dim 128, six at 64), at least two
+    for (int ns = s->head_dim == 128 ? 3 : kTMaxSlots; ns >= 2; --ns) {
+      const int tot = s->head_dim == 128 ? t_layout<128>(ns, s->num_groups, rows).total
+                                         : t_layout<64>(ns, s->num_groups, rows).total;
+      if (tot <= kSmemLimit) {
+        pl->nslots = ns;
+        pl->smem_bytes = tot;
+        break;
+      }
+    }
+    if (pl->nslots == 0)
+      return set_error(RGD_ERR_UNSUPPORTED, "shape needs more shared memory than an SM has (too many groups?)");
+  }
   auto layout = [&](int nslots, int npref) {
     return s->head_dim == 128 ? smem_layout<128>(nslots, s->num_groups, rows, pl->nq, npref)
                               : smem_layout<64>(nslots, s->num_groups, rows, pl->nq, npref);
   };
-  pl->nslots = 0;
   for (int npref = 2; npref >= 1 && pl->nslots == 0; --npref) {
     for (int ns = kMaxSlots; ns >= (npref > 1 ? 4 : 3); --ns) {
       if (layout(ns, npref).total <= kSmemLimit) {
@@ -1449,7 +1480,7 @@ int make_plan(const rgd_attn_shape* s, Plan* pl) {
   }
   if (pl->nslots == 0)
     return set_error(RGD_ERR_UNSUPPORTED, "shape needs more shared memory than an SM has (too many groups?)");
-  pl->smem = layout(pl->nslots, pl->npref);
+  if (!pl->transposed) pl->smem_bytes = layout(pl->nslots, pl->npref).total;
   auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
   const size_t n_part = (size_t)pl->C + pl->J - 1;  // partial-result slots
   // The job counters come first, in an area of at least kTicketSlots counters
@@ -1496,7 +1527,18 @@ int launch_attn(const CUtensorMap& tmK, const CUtensorMap& tmV, const AttnParams
                 cudaStream_t st) {
   static bool done = false;
   if (int rc = ensure_smem(attn_tc_kernel<D, R>, kSmemLimit, &done)) return rc;
-  attn_tc_kernel<D, R><<<pl.C, Roles<R>::kThreads, pl.smem.total, st>>>(tmK, tmV, p);
+  attn_tc_kernel<D, R><<<pl.C, Roles<R>::kThreads, pl.smem_bytes, st>>>(tmK, tmV, p);
+  if (cudaError_t e = cudaGetLastError(); e != cudaSuccess) return cuda_error(e, "attention launch");
+  return RGD_OK;
+}
+
+// The transposed attention kernel (jobs of at most 32 queries) for one head dim.
+template <int D>
+int launch_attn_t(const CUtensorMap& tmK, const CUtensorMap& tmV, const AttnParams& p, const Plan& pl,
+                  cudaStream_t st) {
+  static bool done = false;
+  if (int rc = ensure_smem(attn_t_kernel<D>, kSmemLimit, &done)) return rc;
+  attn_t_kernel<D><<<pl.C, kTThreads, pl.smem_bytes, st>>>(tmK, tmV, p);
   if (cudaError_t e = cudaGetLastError(); e != cudaSuccess) return cuda_error(e, "attention launch");
   return RGD_OK;
 }
@@ -1561,7 +1603,9 @@ extern "C" int rgd_prefix_decode_attn(const rgd_attn_shape* shape, const rgd_bf1
   const int qpc = (pl.nq + 31) / 32;
   const int R = qpc == 1 ? 4 : qpc == 2 ? 2 : 1;  // copies of the queries in the TMEM lanes
   int rc = RGD_OK;
-  if (s.head_dim == 128) {
+  if (pl.transposed) {
+    rc = s.head_dim == 128 ? launch_attn_t<128>(tmK, tmV, p, pl, st) : launch_attn_t<64>(tmK, tmV, p, pl, st);
+  } else if (s.head_dim == 128) {
     rc = R == 4 ? launch_attn<128, 4>(tmK, tmV, p, pl, st)
        : R == 2 ? launch_attn<128, 2>(tmK, tmV, p, pl, st)
                 : launch_attn<128, 1>(tmK, tmV, p, pl, st);
