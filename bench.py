@@ -24,7 +24,6 @@ import argparse
 import hashlib
 import json
 import os
-import re
 import statistics
 import subprocess
 import sys
@@ -74,23 +73,27 @@ def algorithmic_bytes(case):
     return attn, head
 
 
+# DRAM traffic of one attention launch on the Llama-3-8B-shaped step
+# (dram__bytes_read.sum + dram__bytes_write.sum), from one ncu capture of the
+# kernel sources whose hash is given (profiles/attn_t_kernel_llama8b.md has the
+# command); reported only while those sources are unchanged, else null.
+ATTN_TRAFFIC = {"sources_sha256": "cc900676a0ff", "bytes_per_launch": 120529920}
+ATTN_SOURCES = ("attention.cu", "attention_t.cuh")
+
+
 def _kernel_hash():
-    src = os.path.join(ROOT, "paper_2607_20791_gb300", "csrc", "attention.cu")
-    return hashlib.sha256(open(src, "rb").read()).hexdigest()[:12]
+    h = hashlib.sha256()
+    for f in ATTN_SOURCES:
+        h.update(open(os.path.join(ROOT, "paper_2607_20791_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:12]
 
 
 def _profiled_traffic():
-    """Per-launch DRAM bytes of the attention kernel from the committed ncu summary,
-    if it was taken on the current kernel source (else None)."""
-    path = os.path.join(ROOT, "profiles", "attn_tc_kernel_llama8b.md")
-    try:
-        text = open(path).read()
-    except OSError:
+    """Per-launch DRAM bytes of the attention kernel recorded above, if they
+    were taken on the current kernel sources (else None)."""
+    if ATTN_TRAFFIC["bytes_per_launch"] is None or ATTN_TRAFFIC["sources_sha256"] != _kernel_hash():
         return None
-    m = re.search(r"traffic_bytes_per_launch:\s*([0-9]+)\s*\(attention\.cu sha256 ([0-9a-f]+)\)", text)
-    if not m or m.group(2) != _kernel_hash():
-        return None
-    return int(m.group(1))
+    return int(ATTN_TRAFFIC["bytes_per_launch"])
 
 
 class ClockSampler:
@@ -835,12 +838,12 @@ def run_ours(args):
             "step_hbm_gbs": step_gbs, "step_hbm_frac": step_gbs / peak,
             "step_algorithmic_bytes": step_bytes,
             "kernels_ms": {"attention": mean_attn, "sample_head_with_gate": mean_hg},
-            "roofline": {"bound": "hbm", "kernel": "attn_tc_kernel<128, 4>", "achieved": attn_gbs,
+            "roofline": {"bound": "hbm", "kernel": "attn_t_kernel<128>", "achieved": attn_gbs,
                          "peak": peak, "unit": "GB/s", "frac": attn_gbs / peak, "traffic": traffic,
-                         "traffic_source": ("ncu capture of this kernel source (dram bytes read + written per "
-                                            "launch), recorded in profiles/attn_tc_kernel_llama8b.md"
+                         "traffic_source": ("one ncu capture of these kernel sources (dram bytes read + written per "
+                                            "launch), recorded in bench.py with the sources' hash"
                                             if traffic is not None else
-                                            "none: no ncu capture of the current kernel source"),
+                                            "none: no ncu capture of the current kernel sources"),
                          "algorithmic_bytes": attn_bytes, "peak_source": peak_kind},
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
