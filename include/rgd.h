@@ -333,10 +333,14 @@ int rgd_decode_step(const rgd_attn_shape* shape, const rgd_bf16* q, const rgd_bf
  *                  a*), -1 when none (probe discarded or already ended)
  *   mass_out       device float [groups] or NULL: m when the soft branch ran,
  *                  else -1
- * State and row_active as for rgd_probe_gate.  m is accumulated in fp32 (the
- * decision can differ from exact arithmetic only when m is within ~1e-6
- * relative of rho).  RGD_ERR_UNSUPPORTED when a trie node has more than 2047
- * children.  One kernel on `stream`, one block per group. */
+ * State and row_active as for rgd_probe_gate.  m is accumulated in fp32 with
+ * e^x taken as 2^(x log2 e) by the SFU (the decision can differ from exact
+ * arithmetic only when m is within ~1e-5 relative of rho).  dev_status (may
+ * be NULL) gets RGD_DEV_WAIT_TIMEOUT when a bounded wait on a copy of the
+ * logits gave up; that step's outputs are then not valid.
+ * RGD_ERR_UNSUPPORTED when a trie node has more than 2047 children.  One
+ * kernel on `stream`: a cluster of 6 blocks per group, each block reading a
+ * sixth of the probe row. */
 int rgd_soft_gate(const rgd_trie* trie, int32_t groups, int32_t rows_per_group, int32_t vocab, int32_t dtype,
                   const void* probe_logits, int64_t row_stride, int32_t top_k, float rho, int32_t c,
                   int32_t eos_token, int32_t max_len, rgd_gate_state* state, uint8_t* row_active,

@@ -8,9 +8,13 @@
 // the trie before that is incompatible.  The hard gate of Alg. 1 applies the
 // predicate after every greedy probe token (the cap c does not change the
 // outcome of the hard gate).
+#include <cooperative_groups.h>
+
 #include <algorithm>
+#include <climits>
 #include <cmath>
 #include <map>
+#include <mutex>
 #include <vector>
 
 #include "common.h"
@@ -18,6 +22,7 @@
 #include "trie.cuh"
 
 namespace rgd {
+namespace cg = cooperative_groups;
 namespace {
 
 __global__ void gate_state_init_kernel(rgd_gate_state* st, int32_t groups) {
@@ -66,23 +71,49 @@ __global__ void probe_gate_kernel(TrieView t, int32_t groups, int32_t rows_per_g
 // the stop token, which d(q) drops -- are found, and if their probability
 // mass m reaches rho the most probable of them is appended instead.
 //
-// One block per group.  Pass 1 reads the probe's logits once: the maximum, its
-// lowest index (y) and the softmax normaliser Z (per-thread online sums).  The
-// soft branch then sorts the compatible candidates by logit in shared memory
-// (bitonic sort of (logit, token) keys); their ranks grow along that order,
-// so a binary search over it, one pass over the logits (from L2) per probed
-// candidate, finds how many of them are in the top K.
+// One thread-block cluster of kSoftCluster CTAs per group, each CTA taking an
+// equal contiguous share of the probe's logits, copied into shared memory in
+// chunks by bulk copies issued before anything else.  While they are in
+// flight, the children of the probe's trie node (token, node, confirm flag)
+// are read into shared memory -- every trie lookup of the step is then a
+// shared-memory scan -- and, when the soft branch can be taken at this step,
+// the candidates' keys (logit, token) and the kProbe best of them.  A
+// candidate's rank -- the number of logits above it -- grows along the
+// candidates' order, so the candidates in the top K are a prefix of that
+// order.  The pass finds the maximum, its lowest index (y) and the softmax
+// normaliser Z and counts the logits above each of the kProbe best
+// candidates, which settles the prefix unless all of them are in the top K;
+// then the candidates are sorted (bitonic, in shared memory) and a binary
+// search over the rest, one more pass over the logits (from L2) per probed
+// candidate, finishes it.  After each pass every CTA pushes its partial
+// results into every CTA's shared memory and all of them combine the same
+// values in the same order, so every CTA takes the same decisions; CTA 0
+// writes the step's outcome.  The kernel runs once per decode step behind
+// kernels that sweep L2, so its own instructions are fetched cold: its loops
+// stay rolled, which keeps the code it runs short.
 constexpr int kSoftThreads = 512;
-constexpr int kMaxCand = 2048;  // a node's children + the stop token, sorted in shared memory
+constexpr int kSoftCluster = 6;
+constexpr int kMaxCand = 2048;  // a node's children + the stop token (a power of two: the sort's padding)
+constexpr int kProbe = 4;       // candidates whose ranks the first pass counts
+constexpr int kSoftChunk = 32768;  // bytes of logits per bulk copy
+constexpr int kSoftStages = 3;     // chunk buffers
+
+struct SoftPart {  // one CTA's share of the first pass
+  float m, z;
+  int32_t mi;
+  int32_t c[kProbe];
+};
 
 struct SoftShared {
-  uint64_t key[kMaxCand];
-  float red_m[kSoftThreads / 32], red_z[kSoftThreads / 32];
-  int32_t red_i[kSoftThreads / 32];
-  int32_t cnt[1];
-  rgd_gate_state s;
-  float M, Z, mass;
-  int32_t y, mode, ncand, n_in;
+  uint64_t key[kMaxCand];       // slot k < nc: child k; slot nc: the stop token (no candidate: ~0)
+  int32_t slot_tok[kMaxCand];   // child k: its token, the node it leads to, that node's confirm flag
+  int32_t slot_node[kMaxCand];
+  uint8_t slot_conf[kMaxCand];
+  SoftPart part[kSoftCluster * kSoftThreads / 32];  // first pass, slot = CTA rank x warps + warp
+  int32_t cnt[2][kSoftCluster];  // search passes, slot = CTA rank, by pass parity
+  int32_t cnt_cta;
+  uint64_t full[kSoftStages];    // chunk buffer s holds its chunk
+  int32_t ncand;
 };
 
 template <typename LT>
@@ -109,43 +140,62 @@ __device__ __forceinline__ float vec_elem<uint16_t>(const uint4& w, int e) {
   return __uint_as_float((e & 1) ? (u & 0xffff0000u) : (u << 16));
 }
 
-// Calls f(logit, index) for this thread's share of a row, in increasing index
-// order, with kBatchLoads loads in flight: 16-byte vectors when the row is
-// 16-byte aligned (then the few elements past the last whole vector, one per
-// thread, come last), else single elements.
-template <int kThreads, int kBatchLoads, typename LT, typename F>
-__device__ __forceinline__ void scan_row(const LT* row, int32_t vocab, bool vec, F&& f) {
+// Calls f(logit, index) for this thread's share of part `part` (of nparts
+// equal contiguous parts) of a row, in increasing index order: 16-byte
+// vectors when the row is 16-byte aligned (the few elements past the last
+// whole vector, one per thread, go to the last part and come last), else
+// single elements.  Every thread calls between() once, after its first batch
+// of loads is issued and before any f (between() may hold block barriers).
+template <int kThreads, int kBatchLoads, typename LT, typename F, typename B>
+__device__ __forceinline__ void scan_row(const LT* row, int32_t vocab, bool vec, int part, int nparts, F&& f,
+                                         B&& between) {
   constexpr int E = 16 / (int)sizeof(LT);
   const int tid = threadIdx.x;
   if (vec) {
     const int32_t nvec = vocab / E;
+    const int32_t lo = (int32_t)((int64_t)nvec * part / nparts), hi = (int32_t)((int64_t)nvec * (part + 1) / nparts);
     const uint4* rv = reinterpret_cast<const uint4*>(row);
-    for (int32_t v0 = tid; v0 < nvec; v0 += kBatchLoads * kThreads) {
-      uint4 w[kBatchLoads];
+    uint4 w[kBatchLoads];
+    int32_t v0 = lo + tid;
 #pragma unroll
-      for (int b = 0; b < kBatchLoads; ++b)
-        if (v0 + b * kThreads < nvec) w[b] = __ldg(rv + v0 + b * kThreads);
+    for (int b = 0; b < kBatchLoads; ++b)
+      if (v0 + b * kThreads < hi) w[b] = __ldg(rv + v0 + b * kThreads);
+    between();
+    for (;;) {
 #pragma unroll
       for (int b = 0; b < kBatchLoads; ++b) {
         const int32_t vi = v0 + b * kThreads;
-        if (vi >= nvec) break;
+        if (vi >= hi) break;
 #pragma unroll
         for (int e = 0; e < E; ++e) f(vec_elem<LT>(w[b], e), vi * E + e);
       }
-    }
-    const int32_t i = nvec * E + tid;
-    if (i < vocab) f(logit_at<LT>(row, i), i);
-  } else {
-    for (int32_t i0 = tid; i0 < vocab; i0 += kBatchLoads * kThreads) {
-      float v[kBatchLoads];
+      v0 += kBatchLoads * kThreads;
+      if (v0 >= hi) break;
 #pragma unroll
       for (int b = 0; b < kBatchLoads; ++b)
-        if (i0 + b * kThreads < vocab) v[b] = logit_at<LT>(row, i0 + b * kThreads);
+        if (v0 + b * kThreads < hi) w[b] = __ldg(rv + v0 + b * kThreads);
+    }
+    const int32_t i = nvec * E + tid;
+    if (part == nparts - 1 && i < vocab) f(logit_at<LT>(row, i), i);
+  } else {
+    const int32_t lo = (int32_t)((int64_t)vocab * part / nparts), hi = (int32_t)((int64_t)vocab * (part + 1) / nparts);
+    float v[kBatchLoads];
+    int32_t i0 = lo + tid;
+#pragma unroll
+    for (int b = 0; b < kBatchLoads; ++b)
+      if (i0 + b * kThreads < hi) v[b] = logit_at<LT>(row, i0 + b * kThreads);
+    between();
+    for (;;) {
 #pragma unroll
       for (int b = 0; b < kBatchLoads; ++b) {
-        if (i0 + b * kThreads >= vocab) break;
+        if (i0 + b * kThreads >= hi) break;
         f(v[b], i0 + b * kThreads);
       }
+      i0 += kBatchLoads * kThreads;
+      if (i0 >= hi) break;
+#pragma unroll
+      for (int b = 0; b < kBatchLoads; ++b)
+        if (i0 + b * kThreads < hi) v[b] = logit_at<LT>(row, i0 + b * kThreads);
     }
   }
 }
@@ -163,97 +213,309 @@ __device__ __forceinline__ float key_logit(uint64_t k) {
 }
 
 // (v, i) ranks above (w, j): a larger logit, or the same logit and a lower index.
-__device__ __forceinline__ bool above(float v, int64_t i, float w, int64_t j) { return v > w || (v == w && i < j); }
+__device__ __forceinline__ bool above(float v, int32_t i, float w, int32_t j) { return v > w || (v == w && i < j); }
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+// Online softmax state (m, z, mi): the maximum logit seen, z = sum e^(l - m)
+// over the logits seen (e^x = 2^(x log2 e), by the SFU), and the lowest index
+// of the maximum.  Merges (om, oz, oi).
+__device__ __forceinline__ void merge_mz(float& m, float& z, int32_t& mi, float om, float oz, int32_t oi) {
+  const float nm = fmaxf(m, om);
+  if (nm != -INFINITY) z = z * ex2_approx((m - nm) * kLog2e) + oz * ex2_approx((om - nm) * kLog2e);
+  if (om > m || (om == m && oi < mi)) mi = oi;
+  m = nm;
+}
+
+// The SoftParts of a warp's lanes, and n more from shared memory (n a multiple
+// of 32: lane l folds parts[l], parts[l + 32], ...), merged in a fixed order;
+// every lane returns lane 0's result.  One rolled loop, not inlined: every
+// merge of the step runs the same few lines of code.
+__device__ __noinline__ SoftPart merge_lanes(SoftPart p, const SoftPart* parts, int n) {
+  const int lane = threadIdx.x & 31;
+  int i = lane, o = 16;
+#pragma unroll 1
+  for (;;) {
+    SoftPart q;
+    if (i < n) {  // (uniform: n is a multiple of 32)
+      q = parts[i];
+      i += 32;
+    } else if (o > 0) {
+      q.m = __shfl_xor_sync(0xffffffffu, p.m, o);
+      q.z = __shfl_xor_sync(0xffffffffu, p.z, o);
+      q.mi = __shfl_xor_sync(0xffffffffu, p.mi, o);
+#pragma unroll
+      for (int k = 0; k < kProbe; ++k) q.c[k] = __shfl_xor_sync(0xffffffffu, p.c[k], o);
+      o >>= 1;
+    } else {
+      break;
+    }
+    merge_mz(p.m, p.z, p.mi, q.m, q.z, q.mi);
+#pragma unroll
+    for (int k = 0; k < kProbe; ++k) p.c[k] += q.c[k];
+  }
+  p.m = __shfl_sync(0xffffffffu, p.m, 0);  // (the lanes may differ in z's rounding)
+  p.z = __shfl_sync(0xffffffffu, p.z, 0);
+  p.mi = __shfl_sync(0xffffffffu, p.mi, 0);
+  return p;
+}
 
 template <typename LT>
-__global__ void __launch_bounds__(kSoftThreads)
+__global__ void __cluster_dims__(kSoftCluster, 1, 1) __launch_bounds__(kSoftThreads, 1)
     soft_gate_kernel(TrieView t, int32_t rows_per_group, int32_t vocab, const LT* __restrict__ logits,
                      int64_t row_stride, bool vec, int32_t top_k, float rho, int32_t c, int32_t eos, int32_t max_len,
                      rgd_gate_state* __restrict__ state, uint8_t* __restrict__ row_active, int32_t* token_out,
-                     float* mass_out) {
+                     float* mass_out, int32_t* dev_status) {
+  constexpr int E = 16 / (int)sizeof(LT);   // logits per 16-byte vector
+  constexpr int kVpc = kSoftChunk / 16;      // vectors per chunk
+  constexpr int kWarps = kSoftThreads / 32;
   __shared__ SoftShared sh;
-  const int g = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  extern __shared__ uint4 soft_buf[];  // kSoftStages chunks
+  cg::cluster_group cluster = cg::this_cluster();
+  const int rank = (int)cluster.block_rank();
+  const int g = blockIdx.x / kSoftCluster, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const LT* row = logits + (int64_t)g * row_stride;
+  // this CTA's share of the row: vectors [lo, lo + nv) when the row is
+  // 16-byte aligned (staged through shared memory), else elements [lo, hi_u)
+  const int32_t nvec = vocab / E;
+  const int32_t n_units = vec ? nvec : vocab;
+  const int32_t lo = (int32_t)((int64_t)n_units * rank / kSoftCluster);
+  const int32_t hi_u = (int32_t)((int64_t)n_units * (rank + 1) / kSoftCluster);
+  const int32_t nv = vec ? hi_u - lo : 0;
+  const int32_t nchunks = (nv + kVpc - 1) / kVpc;
+  const uint4* rv = reinterpret_cast<const uint4*>(row);
+  auto issue = [&](int32_t ck) {  // (thread 0) chunk ck into buffer ck % kSoftStages
+    const uint32_t bytes = (uint32_t)min(kVpc, nv - ck * kVpc) * 16u;
+    uint64_t* bar = &sh.full[ck % kSoftStages];
+    mbar_arrive_expect_tx(bar, bytes);
+    bulk_load(soft_buf + (ck % kSoftStages) * kVpc, rv + lo + ck * kVpc, bytes, bar);
+  };
+  bool timed_out = false;
+  auto wait_chunk = [&](int32_t ck) {  // bounded; a second bounded wait after a timeout
+    uint64_t* bar = &sh.full[ck % kSoftStages];
+    const uint32_t par = (uint32_t)(ck / kSoftStages) & 1u;
+    if (!mbar_wait(bar, par)) {
+      timed_out = true;
+      mbar_wait(bar, par);
+    }
+  };
   if (tid == 0) {
-    sh.s = state[g];
-    sh.mode = 0;
-    sh.mass = -1.f;
+    for (int b = 0; b < kSoftStages; ++b) mbar_init(&sh.full[b], 1);
+    fence_mbar_init();
+    for (int32_t ck = 0; ck < min(kSoftStages, nchunks); ++ck) issue(ck);
+    sh.ncand = 0;
   }
+  // Every thread reads the state and takes the same decisions from it: the
+  // kernel has no section where one warp works while the others wait.
+  const rgd_gate_state s0 = state[g];
   __syncthreads();
-  if (sh.s.done) {  // (uniform) nothing to consume
+  if (s0.done) {  // (uniform over the cluster) nothing to consume
     if (tid == 0) {
-      token_out[g] = -1;
-      if (mass_out) mass_out[g] = -1.f;
+      for (int32_t ck = 0; ck < min(kSoftStages, nchunks); ++ck) wait_chunk(ck);  // (no copy outlives the CTA)
+      if (timed_out && dev_status) atomicOr(dev_status, RGD_DEV_WAIT_TIMEOUT);
+      if (rank == 0) {
+        token_out[g] = -1;
+        if (mass_out) mass_out[g] = -1.f;
+      }
     }
     return;
   }
-  // ---- pass 1: maximum, its lowest index, and Z = sum exp(l - max) ----
+  cluster_arrive_relaxed();  // (waited for before the first push into another CTA)
+
+  // ---- while the first chunks are in flight: the node's children (needed
+  // unless the probe is confirmed) and, when the soft branch can be taken at
+  // this step (the first c steps), the candidates' keys and the kProbe best ----
+  const bool gather = !s0.confirmed;
+  const bool maybe_soft = gather && s0.steps < c;
+  int32_t cb = 0, nc = 0;
+  if (gather) {
+    cb = __ldg(t.child_begin + s0.node);
+    nc = __ldg(t.child_begin + s0.node + 1) - cb;
+  }
+  const int32_t nslot = maybe_soft ? nc + 1 : nc;
+  {
+    int32_t mine = 0;
+    for (int32_t k = tid; k < nslot; k += kSoftThreads) {
+      int32_t a = eos;
+      if (k < nc) {
+        a = __ldg(t.child_tok + cb + k);
+        const int32_t nd = __ldg(t.child_node + cb + k);
+        sh.slot_tok[k] = a;
+        sh.slot_node[k] = nd;
+        sh.slot_conf[k] = __ldg(t.confirm + nd);
+      }
+      if (maybe_soft) {
+        const bool ok = a >= 0 && a < vocab && (k == nc || a != eos);
+        sh.key[k] = ok ? rank_key(logit_at<LT>(row, a), a) : ~0ull;
+        mine += ok ? 1 : 0;
+      }
+    }
+    if (mine) atomicAdd(&sh.ncand, mine);
+  }
+  __syncthreads();
+  const int32_t n = sh.ncand;        // candidates
+  const int32_t hi = min(n, top_k);  // only the first hi of them can be in the top K
+  const int32_t np_ = min(hi, kProbe);
+  // the np_ smallest keys (every warp finds them: one warp-wide minimum each;
+  // keys are distinct); their logits and tokens probe the pass
+  float pv[kProbe];
+  int32_t pi[kProbe], pc[kProbe];
+  {
+    uint64_t prev = 0;
+#pragma unroll
+    for (int q = 0; q < kProbe; ++q) {
+      uint64_t best = ~0ull;
+      if (q < np_) {
+#pragma unroll 1
+        for (int32_t k = lane; k < nslot; k += 32) {
+          const uint64_t key = sh.key[k];
+          if ((q == 0 || key > prev) && key < best) best = key;
+        }
+        const uint32_t bh = __reduce_min_sync(0xffffffffu, (uint32_t)(best >> 32));
+        const uint32_t bl = __reduce_min_sync(0xffffffffu, (uint32_t)(best >> 32) == bh ? (uint32_t)best : ~0u);
+        best = ((uint64_t)bh << 32) | bl;
+      }
+      prev = best;
+      pv[q] = q < np_ ? key_logit(best) : INFINITY;  // (nothing ranks above +inf at index 0)
+      pi[q] = q < np_ ? (int32_t)(uint32_t)best : 0;
+      pc[q] = 0;
+    }
+  }
+  const float p_min = np_ > 0 ? pv[np_ - 1] : INFINITY;  // only a logit >= this can rank above a probe
+
+  // ---- the pass: maximum, its lowest index, z = sum e^(l - m), probe ranks ----
   float m = -INFINITY, z = 0.f;
   int32_t mi = 0x7fffffff;
-  scan_row<kSoftThreads, 8, LT>(row, vocab, vec, [&](float v, int32_t i) {
-    if (v > m) {  // indices grow along a thread: strict > keeps the lowest
-      z = (m == -INFINITY) ? 1.f : z * expf(m - v) + 1.f;
+  auto probe_counts = [&](float v, int32_t i) {
+#pragma unroll
+    for (int q = 0; q < kProbe; ++q) pc[q] += above(v, i, pv[q], pi[q]) ? 1 : 0;
+  };
+  auto one = [&](float v, int32_t i) {  // a single logit (indices grow along a thread)
+    if (v > m) {
+      z = (m == -INFINITY) ? 0.f : z * ex2_approx((m - v) * kLog2e);
       m = v;
       mi = i;
-    } else if (m != -INFINITY) {  // (with m = -inf, v is -inf too and adds nothing)
-      z += expf(v - m);
     }
-  });
+    if (m != -INFINITY) z += ex2_approx(fmaf(v, kLog2e, -m * kLog2e));
+    if (v >= p_min) probe_counts(v, i);
+  };
+  if (vec) {
+    for (int32_t ck = 0; ck < nchunks; ++ck) {
+      wait_chunk(ck);
+      const uint4* buf = soft_buf + (ck % kSoftStages) * kVpc;
+      const int32_t cnt = min(kVpc, nv - ck * kVpc), base = lo + ck * kVpc;
+      // this thread's vectors of the chunk: their maximum first, so that the
+      // running maximum moves at most once per chunk
+      float bm = -INFINITY;
+#pragma unroll 1
+      for (int32_t k = tid; k < cnt; k += kSoftThreads) {
+        const uint4 x = buf[k];
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float om = __shfl_xor_sync(0xffffffffu, m, o), oz = __shfl_xor_sync(0xffffffffu, z, o);
-    const int32_t oi = __shfl_xor_sync(0xffffffffu, mi, o);
-    const float nm = fmaxf(m, om);
-    z = (m == -INFINITY ? 0.f : z * expf(m - nm)) + (om == -INFINITY ? 0.f : oz * expf(om - nm));
-    if (om > m || (om == m && oi < mi)) mi = oi;
-    m = nm;
-  }
-  if (lane == 0) {
-    sh.red_m[warp] = m;
-    sh.red_z[warp] = z;
-    sh.red_i[warp] = mi;
-  }
-  __syncthreads();
-  if (tid == 0) {
-    float M = sh.red_m[0], Z = sh.red_z[0];
-    int32_t A = sh.red_i[0];
-    for (int w = 1; w < kSoftThreads / 32; ++w) {
-      const float om = sh.red_m[w], oz = sh.red_z[w];
-      const float nm = fmaxf(M, om);
-      Z = (M == -INFINITY ? 0.f : Z * expf(M - nm)) + (om == -INFINITY ? 0.f : oz * expf(om - nm));
-      if (om > M || (om == M && sh.red_i[w] < A)) A = sh.red_i[w];
-      M = nm;
-    }
-    sh.M = M;
-    sh.Z = Z;
-    sh.y = A;
-    const rgd_gate_state& s = sh.s;
-    const bool stop = eos >= 0 && A == eos;
-    const bool compatible = s.confirmed || find_child(t, s.node, A) >= 0;
-    sh.mode = (s.steps >= c || stop || compatible) ? 1 : 2;  // 1: the hard step with y; 2: the soft branch
-    if (sh.mode == 2) {
-      // the candidates: children of the node (and the stop token) inside the vocabulary
-      const int32_t b = __ldg(t.child_begin + s.node), e = __ldg(t.child_begin + s.node + 1);
-      int32_t n = 0;
-      for (int32_t k = b; k < e; ++k) {
-        const int32_t a = __ldg(t.child_tok + k);
-        if (a >= 0 && a < vocab && a != eos) sh.key[n++] = rank_key(logit_at<LT>(row, a), a);
+        for (int e = 0; e < E; ++e) bm = fmaxf(bm, vec_elem<LT>(x, e));
       }
-      if (eos >= 0 && eos < vocab) sh.key[n++] = rank_key(logit_at<LT>(row, eos), eos);
-      sh.ncand = n;
+      if (bm > m) {  // the lowest index of bm here (indices grow along k, then e)
+        int32_t bi = 0x7fffffff;
+#pragma unroll 1
+        for (int32_t k = tid; k < cnt && bi == 0x7fffffff; k += kSoftThreads) {
+          const uint4 x = buf[k];
+#pragma unroll
+          for (int e = E - 1; e >= 0; --e)
+            if (vec_elem<LT>(x, e) == bm) bi = (base + k) * E + e;
+        }
+        z = (m == -INFINITY) ? 0.f : z * ex2_approx((m - bm) * kLog2e);
+        m = bm;
+        mi = bi;
+      }
+      // z, and the probes for the few logits at or above the weakest one
+      if (m != -INFINITY) {
+        const float ml = m * kLog2e;
+#pragma unroll 1
+        for (int32_t k = tid; k < cnt; k += kSoftThreads) {
+          const uint4 x = buf[k];
+          float z0 = 0.f, z1 = 0.f;
+#pragma unroll
+          for (int e = 0; e < E; e += 2) {
+            const float v0 = vec_elem<LT>(x, e), v1 = vec_elem<LT>(x, e + 1);
+            z0 += ex2_approx(fmaf(v0, kLog2e, -ml));
+            z1 += ex2_approx(fmaf(v1, kLog2e, -ml));
+            if (v0 >= p_min) probe_counts(v0, (base + k) * E + e);
+            if (v1 >= p_min) probe_counts(v1, (base + k) * E + e + 1);
+          }
+          z += z0 + z1;
+        }
+      } else if (bm >= p_min) {  // (every logit so far is -inf, and so is a probed candidate)
+#pragma unroll 1
+        for (int32_t k = tid; k < cnt; k += kSoftThreads) {
+          const uint4 x = buf[k];
+#pragma unroll
+          for (int e = 0; e < E; ++e) probe_counts(vec_elem<LT>(x, e), (base + k) * E + e);
+        }
+      }
+      if (ck + kSoftStages < nchunks) {
+        __syncthreads();  // the buffer is free
+        if (tid == 0) issue(ck + kSoftStages);
+      }
     }
+    // the few logits past the last whole vector
+    const int32_t i = nvec * E + tid;
+    if (rank == kSoftCluster - 1 && i < vocab) one(logit_at<LT>(row, i), i);
+  } else {
+    scan_row<kSoftThreads, 8, LT>(row, vocab, false, rank, kSoftCluster, one, [] {});
   }
-  __syncthreads();
-  if (sh.mode == 2) {
-    // ---- sort the candidates (bitonic, padded to a power of two) ----
-    const int32_t n = sh.ncand;
-    int32_t np = 1;
-    while (np < n) np <<= 1;
-    for (int32_t i = n + tid; i < np; i += kSoftThreads) sh.key[i] = ~0ull;
+  if (timed_out && dev_status) atomicOr(dev_status, RGD_DEV_WAIT_TIMEOUT);  // (the outputs are then not valid)
+
+  // ---- every warp's share -> every CTA of the cluster ----
+  {
+    SoftPart p;
+    p.m = m;
+    p.z = z;
+    p.mi = mi;
+#pragma unroll
+    for (int q = 0; q < kProbe; ++q) p.c[q] = pc[q];
+    p = merge_lanes(p, nullptr, 0);
+    cluster_wait();  // every CTA of the cluster has started
+    if (lane < kSoftCluster) cluster.map_shared_rank(&sh, lane)->part[rank * kWarps + warp] = p;
+  }
+  cluster.sync();  // every warp's share is in every CTA's shared memory
+  // ---- the same combination, in the same order, in every warp of the cluster ----
+  SoftPart all;
+  all.m = -INFINITY;
+  all.z = 0.f;
+  all.mi = 0x7fffffff;
+#pragma unroll
+  for (int q = 0; q < kProbe; ++q) all.c[q] = 0;
+  all = merge_lanes(all, sh.part, kSoftCluster * kWarps);
+  const int32_t y = all.mi;
+  // the children labelled y and a* (the best candidate), if any
+  const int32_t a_star = np_ > 0 ? pi[0] : -1;
+  int32_t sy = -1, sa = -1;
+#pragma unroll 1
+  for (int32_t k = lane; k < nc; k += 32) {
+    const int32_t tk = sh.slot_tok[k];
+    if (tk == y) sy = k;  // (a node's children have distinct tokens)
+    if (tk == a_star) sa = k;
+  }
+  sy = __reduce_max_sync(0xffffffffu, sy);
+  sa = __reduce_max_sync(0xffffffffu, sa);
+  const bool stop = eos >= 0 && y == eos;
+  const bool compatible = s0.confirmed || sy >= 0;
+  const bool soft = !(s0.steps >= c || stop || compatible);  // else the hard step with y
+  // the probed candidates in the top K (a prefix: ranks grow along the order)
+  int32_t n_in = 0;
+  if (soft)
+    while (n_in < np_ && all.c[n_in] < top_k) ++n_in;
+  if (soft && n_in == np_ && np_ < hi) {
+    // ---- the rest: sort the candidates (bitonic, padded to a power of two;
+    // the first np_ are the probed ones), then a binary search over
+    // candidates np_ .. hi - 1, one comparison per logit per probed
+    // candidate (every thread of the cluster takes the same steps) ----
+    int32_t np2 = 1;
+    while (np2 < nslot) np2 <<= 1;
+    for (int32_t i = nslot + tid; i < np2; i += kSoftThreads) sh.key[i] = ~0ull;
     __syncthreads();
-    for (int32_t k = 2; k <= np; k <<= 1) {
+    for (int32_t k = 2; k <= np2; k <<= 1) {
       for (int32_t j = k >> 1; j > 0; j >>= 1) {
-        for (int32_t i = tid; i < np; i += kSoftThreads) {
+        for (int32_t i = tid; i < np2; i += kSoftThreads) {
           const int32_t ij = i ^ j;
           if (ij > i) {
             const uint64_t a = sh.key[i], b2 = sh.key[ij];
@@ -266,46 +528,66 @@ __global__ void __launch_bounds__(kSoftThreads)
         __syncthreads();
       }
     }
-    // ---- how many of the sorted candidates are in the top K: their ranks
-    // grow along the order, so a binary search, one candidate per pass (each
-    // pass one comparison per logit, the logits read from L2) ----
-    int32_t lo = 0, hi = min(n, top_k);
-    while (lo < hi) {  // (lo, hi are the same in every thread)
-      const int32_t mid = (lo + hi) >> 1;
+    int32_t lo_c = np_, hi_c = hi;
+    for (int pass = 0; lo_c < hi_c; ++pass) {
+      const int32_t mid = (lo_c + hi_c) >> 1;
       const uint64_t key = sh.key[mid];
       const float cv = key_logit(key);
       const int32_t ci = (int32_t)(uint32_t)key;
-      if (tid == 0) sh.cnt[0] = 0;
+      if (tid == 0) sh.cnt_cta = 0;
       __syncthreads();
       int32_t cnt = 0;
-      scan_row<kSoftThreads, 8, LT>(row, vocab, vec, [&](float v, int32_t i) { cnt += above(v, i, cv, ci) ? 1 : 0; });
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
-      if (lane == 0 && cnt) atomicAdd(&sh.cnt[0], cnt);
+      scan_row<kSoftThreads, 8, LT>(
+          row, vocab, vec, rank, kSoftCluster, [&](float v, int32_t i) { cnt += above(v, i, cv, ci) ? 1 : 0; },
+          [] {});
+      cnt = __reduce_add_sync(0xffffffffu, cnt);
+      if (lane == 0 && cnt) atomicAdd(&sh.cnt_cta, cnt);
       __syncthreads();
-      if (sh.cnt[0] < top_k) lo = mid + 1;
-      else hi = mid;
-      __syncthreads();  // (sh.cnt is reset in the next pass)
+      // CTA r's slot of this pass's parity is next written two passes on,
+      // after every CTA has passed the next cluster barrier (and read this one)
+      if (warp == 0 && lane < kSoftCluster) cluster.map_shared_rank(&sh, lane)->cnt[pass & 1][rank] = sh.cnt_cta;
+      cluster.sync();
+      int32_t total = 0;
+      for (int r = 0; r < kSoftCluster; ++r) total += sh.cnt[pass & 1][r];
+      if (total < top_k) lo_c = mid + 1;
+      else hi_c = mid;
     }
-    if (tid == 0) {
-      sh.n_in = lo;
-      float mass = 0.f;
-      for (int k = 0; k < lo; ++k) mass += expf(key_logit(sh.key[k]) - sh.M) / sh.Z;
-      sh.mass = mass;
-    }
-    __syncthreads();
+    n_in = lo_c;
   }
-  if (tid != 0) return;
-  // ---- the step's outcome ----
-  rgd_gate_state s = sh.s;
+  // (no CTA touches another's shared memory after the last cluster barrier)
+  if (warp != 0 || rank != 0) return;
+  // ---- the step's outcome (warp 0 of CTA 0) ----
+  float mass = -1.f;
+  if (soft) {
+    // m = the probability mass of the candidates in the top K
+    const float ml = all.m * kLog2e;
+    float part = 0.f;
+    for (int32_t k = lane; k < n_in; k += 32) {
+      float l = 0.f;
+#pragma unroll
+      for (int q = 0; q < kProbe; ++q)
+        if (k == q) l = pv[q];
+      if (k >= kProbe) l = key_logit(sh.key[k]);
+      part += ex2_approx(fmaf(l, kLog2e, -ml));
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+    mass = part / all.z;
+  }
+  if (lane != 0) return;
+  rgd_gate_state s = s0;
+  auto child = [&](int32_t tok) {  // the gathered children: tok is y or a*
+    const int32_t k = tok == y ? sy : sa;
+    return k < 0 ? make_int2(-1, 0) : make_int2(sh.slot_node[k], (int)sh.slot_conf[k]);
+  };
   const bool root_has_children = __ldg(t.child_begin + 1) > __ldg(t.child_begin);
   int32_t tok = -1;
-  if (sh.mode == 1) {
-    tok = sh.y;
-    consume_token(t, s, tok, eos, max_len, root_has_children);
-  } else if (sh.n_in > 0 && sh.mass >= rho) {
-    tok = (int32_t)(uint32_t)sh.key[0];  // a*: the most probable compatible token
-    consume_token(t, s, tok, eos, max_len, root_has_children);
+  if (!soft) {
+    tok = y;
+    consume_token_with(s, tok, eos, max_len, root_has_children, child);
+  } else if (n_in > 0 && mass >= rho) {
+    tok = a_star;  // the most probable compatible token
+    consume_token_with(s, tok, eos, max_len, root_has_children, child);
   } else {  // no refusal-like alternative with enough mass: discard the probe
     s.decision = RGD_NON_REFUSAL;
     s.decisive_step = s.steps;
@@ -314,7 +596,7 @@ __global__ void __launch_bounds__(kSoftThreads)
   }
   state[g] = s;
   token_out[g] = tok;
-  if (mass_out) mass_out[g] = sh.mode == 2 ? sh.mass : -1.f;
+  if (mass_out) mass_out[g] = soft ? mass : -1.f;
   mask_rows(s, row_active, g, rows_per_group);
 }
 
@@ -454,9 +736,9 @@ extern "C" int rgd_soft_gate(const rgd_trie* trie, int32_t groups, int32_t rows_
                              uint8_t* row_active, int32_t* token_out, float* mass_out, int32_t* dev_status,
                              rgd_stream_t stream) {
   clear_error();
-  (void)dev_status;
   RGD_CHECK_ARG(trie != nullptr, "rgd_soft_gate: trie is NULL");
-  RGD_CHECK_ARG(groups >= 0 && rows_per_group >= 1 && vocab >= 1, "rgd_soft_gate: bad groups/rows/vocab");
+  RGD_CHECK_ARG(groups >= 0 && groups <= INT32_MAX / kSoftCluster && rows_per_group >= 1 && vocab >= 1,
+                "rgd_soft_gate: bad groups/rows/vocab");
   RGD_CHECK_ARG(dtype == RGD_F32 || dtype == RGD_BF16, "rgd_soft_gate: dtype must be RGD_F32 or RGD_BF16");
   RGD_CHECK_ARG(row_stride >= vocab, "rgd_soft_gate: row_stride < vocab");
   RGD_CHECK_ARG(top_k >= 1 && c >= 0 && max_len >= 1, "rgd_soft_gate: need top_k >= 1, c >= 0, max_len >= 1");
@@ -471,16 +753,20 @@ extern "C" int rgd_soft_gate(const rgd_trie* trie, int32_t groups, int32_t rows_
   cudaStream_t st = (cudaStream_t)stream;
   const int es = dtype == RGD_F32 ? 4 : 2;
   const bool vec = aligned16(probe_logits) && (row_stride * es) % 16 == 0;  // 16-byte vector loads
+  constexpr int kDyn = kSoftStages * kSoftChunk;  // chunk buffers (dynamic shared memory)
+  static std::once_flag attr_once;
+  std::call_once(attr_once, [] {
+    cudaFuncSetAttribute(soft_gate_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, kDyn);
+    cudaFuncSetAttribute(soft_gate_kernel<uint16_t>, cudaFuncAttributeMaxDynamicSharedMemorySize, kDyn);
+  });
   if (dtype == RGD_F32)
-    soft_gate_kernel<float><<<groups, kSoftThreads, 0, st>>>(tv, rows_per_group, vocab,
-                                                              static_cast<const float*>(probe_logits), row_stride,
-                                                              vec, top_k, rho, c, eos_token, max_len, state, row_active,
-                                                              token_out, mass_out);
+    soft_gate_kernel<float><<<groups * kSoftCluster, kSoftThreads, kDyn, st>>>(
+        tv, rows_per_group, vocab, static_cast<const float*>(probe_logits), row_stride, vec, top_k, rho, c, eos_token,
+        max_len, state, row_active, token_out, mass_out, dev_status);
   else
-    soft_gate_kernel<uint16_t><<<groups, kSoftThreads, 0, st>>>(tv, rows_per_group, vocab,
-                                                                 static_cast<const uint16_t*>(probe_logits),
-                                                                 row_stride, vec, top_k, rho, c, eos_token, max_len,
-                                                                 state, row_active, token_out, mass_out);
+    soft_gate_kernel<uint16_t><<<groups * kSoftCluster, kSoftThreads, kDyn, st>>>(
+        tv, rows_per_group, vocab, static_cast<const uint16_t*>(probe_logits), row_stride, vec, top_k, rho, c,
+        eos_token, max_len, state, row_active, token_out, mass_out, dev_status);
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? RGD_OK : cuda_error(e, "soft_gate launch");
 }

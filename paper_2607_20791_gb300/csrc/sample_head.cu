@@ -251,6 +251,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
     }
     return;
   }
+  cluster_arrive_relaxed();  // (waited for before the first push into another CTA)
   const uint8_t* rowp = p.logits + (int64_t)row * p.vocab * V::kSize;
   const int spw = p.spw;
   // warp w of CTA r reads stripes [(8r + w) spw, (8r + w + 1) spw) of the row
@@ -318,6 +319,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
     sh.red_v[warp] = bv;
     sh.red_i[warp] = bi;
   }
+  cluster_wait();  // every CTA of the cluster has started
   __syncthreads();
   if (warp == 0) {
     float v = sh.red_v[0];

@@ -49,9 +49,12 @@ __device__ __forceinline__ int32_t find_child(const TrieView& t, int32_t node, i
 }
 
 // One probe token y (the stop token, or y >= 0) through the hard gate, for a
-// state whose probe has not ended.
-__device__ void consume_token(const TrieView& t, rgd_gate_state& s, int32_t y, int32_t eos, int32_t max_len,
-                              bool root_has_children) {
+// state whose probe has not ended.  child(y) gives the trie edge labelled y
+// out of s.node as {node it leads to, whether that node confirms}, or
+// {-1, 0} when there is none.
+template <typename Child>
+__device__ void consume_token_with(rgd_gate_state& s, int32_t y, int32_t eos, int32_t max_len,
+                                   bool root_has_children, Child&& child) {
   if (eos >= 0 && y == eos) {
     const int32_t step = s.steps++;
     s.done = 1;
@@ -66,15 +69,15 @@ __device__ void consume_token(const TrieView& t, rgd_gate_state& s, int32_t y, i
   const int32_t step = s.steps++;
   s.length++;
   if (!s.confirmed) {
-    const int32_t e = find_child(t, s.node, y);
-    if (e < 0) {
+    const int2 e = child(y);
+    if (e.x < 0) {
       s.decision = RGD_NON_REFUSAL;
       s.decisive_step = step;
       s.done = 1;
       return;
     }
-    s.node = __ldg(t.child_node + e);
-    if (__ldg(t.confirm + s.node)) {
+    s.node = e.x;
+    if (e.y) {
       s.confirmed = 1;
       if (s.decision == RGD_PENDING) {
         s.decision = RGD_REFUSAL;
@@ -89,6 +92,17 @@ __device__ void consume_token(const TrieView& t, rgd_gate_state& s, int32_t y, i
       s.decisive_step = step;
     }
   }
+}
+
+// consume_token_with, the edge looked up in the trie.
+__device__ __forceinline__ void consume_token(const TrieView& t, rgd_gate_state& s, int32_t y, int32_t eos,
+                                              int32_t max_len, bool root_has_children) {
+  consume_token_with(s, y, eos, max_len, root_has_children, [&](int32_t tok) {
+    const int32_t e = find_child(t, s.node, tok);
+    if (e < 0) return make_int2(-1, 0);
+    const int32_t nd = __ldg(t.child_node + e);
+    return make_int2(nd, (int)__ldg(t.confirm + nd));
+  });
 }
 
 // The gate's row mask: the probe row off once the probe has ended, the sample
