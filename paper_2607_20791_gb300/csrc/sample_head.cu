@@ -199,9 +199,7 @@ struct Shared {
   float cta_sum[kClusterCtas];
   int32_t cta_cnt[kClusterCtas];
   // broadcast within the CTA
-  float row_max;
-  int32_t row_arg;
-  float cut;
+  float theta;  // T ln p_min (thread 0)
 };
 
 // Compensated (Kahan) fp32 running sum: the prefix sums of the draw stay within
@@ -270,6 +268,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
   float u = 0.f, theta = -INFINITY;
   if (tid == 0) {
     if (mp > 0.0f) theta = (float)((double)temp * log((double)mp));
+    sh.theta = theta;  // (read after the first cluster barrier)
     const uint64_t sd = p.seed[row];
     const uint32_t x0 = philox_word0((uint32_t)p.step, (uint32_t)(p.step >> 32), 0u, 0u, (uint32_t)sd,
                                      (uint32_t)(sd >> 32));
@@ -340,32 +339,22 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
   // traffic is writes before a barrier and local reads after it, so no CTA
   // needs to outlive another's reads.)
   cluster.sync();
-  if (warp == 0) {
-    // one lane per CTA of the cluster reads its maximum (the remote loads overlap)
-    float v = -INFINITY;
-    int32_t i = 0x7fffffff;
-    if (lane < kClusterCtas) {
-      v = sh.cta_max[lane];
-      i = sh.cta_arg[lane];
-    }
+  // every warp merges the CTAs' maxima itself (no warp waits on another here)
+  float M = -INFINITY;
+  int32_t A = 0x7fffffff;
+  if (lane < kClusterCtas) {
+    M = sh.cta_max[lane];
+    A = sh.cta_arg[lane];
+  }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, v, o);
-      const int32_t oi = __shfl_xor_sync(0xffffffffu, i, o);
-      if (better(ov, oi, v, i)) {
-        v = ov;
-        i = oi;
-      }
-    }
-    if (lane == 0) {
-      sh.row_max = v;
-      sh.row_arg = i;
-      sh.cut = __fadd_rn(v, theta);  // the min-p cutoff fl32(M + fl32(T ln p_min))
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, M, o);
+    const int32_t oi = __shfl_xor_sync(0xffffffffu, A, o);
+    if (better(ov, oi, M, A)) {
+      M = ov;
+      A = oi;
     }
   }
-  __syncthreads();
-  const float M = sh.row_max;
-  const int32_t A = sh.row_arg;
   const bool greedy = probe || temp == 0.0f;
   const bool bad = !(temp >= 0.0f) || !isfinite(temp) || !(mp >= 0.0f && mp <= 1.0f) || !isfinite(M) ||
                    A >= p.vocab;
@@ -386,7 +375,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kHeadThre
   }
 
   // ---- pass 2: kept weights; the sum of every stripe and of every warp -------
-  const float cut = sh.cut;
+  const float cut = __fadd_rn(M, sh.theta);  // the min-p cutoff fl32(M + fl32(T ln p_min))
   const float kexp = 1.4426950408889634f / temp;
   uint8_t* mask = p.kept_mask ? p.kept_mask + (int64_t)row * p.vocab : nullptr;
   KSum wsum;  // identical in every lane
