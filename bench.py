@@ -77,7 +77,7 @@ def algorithmic_bytes(case):
 # (dram__bytes_read.sum + dram__bytes_write.sum), from one ncu capture of the
 # kernel sources whose hash is given (profiles/attn_t_kernel_llama8b.md has the
 # command); reported only while those sources are unchanged, else null.
-ATTN_TRAFFIC = {"sources_sha256": "cc900676a0ff", "bytes_per_launch": 120529920}
+ATTN_TRAFFIC = {"sources_sha256": "2d8c69d2bd96", "bytes_per_launch": 121424896}
 ATTN_SOURCES = ("attention.cu", "attention_t.cuh")
 
 
@@ -855,7 +855,7 @@ def run_ours(args):
             "step_hbm_gbs": step_gbs, "step_hbm_frac": step_gbs / peak,
             "step_algorithmic_bytes": step_bytes,
             "kernels_ms": {"attention": mean_attn, "sample_head_with_gate": mean_hg},
-            "roofline": {"bound": "hbm", "kernel": "attn_t_kernel<128>", "achieved": attn_gbs,
+            "roofline": {"bound": "hbm", "kernel": "attn_t_kernel<128, 3>", "achieved": attn_gbs,
                          "peak": peak, "unit": "GB/s", "frac": attn_gbs / peak, "traffic": traffic,
                          "traffic_source": ("one ncu capture of these kernel sources (dram bytes read + written per "
                                             "launch), recorded in bench.py with the sources' hash"

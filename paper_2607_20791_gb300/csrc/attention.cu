@@ -1532,15 +1532,26 @@ int launch_attn(const CUtensorMap& tmK, const CUtensorMap& tmV, const AttnParams
   return RGD_OK;
 }
 
-// The transposed attention kernel (jobs of at most 32 queries) for one head dim.
+// The transposed attention kernel (jobs of at most 32 queries) for one head
+// dim and NS softmax sets of 8 queries.
+template <int D, int NS>
+int launch_attn_t_ns(const CUtensorMap& tmK, const CUtensorMap& tmV, const AttnParams& p, const Plan& pl,
+                     cudaStream_t st) {
+  static bool done = false;
+  if (int rc = ensure_smem(attn_t_kernel<D, NS>, kSmemLimit, &done)) return rc;
+  attn_t_kernel<D, NS><<<pl.C, t_threads<NS>(), pl.smem_bytes, st>>>(tmK, tmV, p);
+  if (cudaError_t e = cudaGetLastError(); e != cudaSuccess) return cuda_error(e, "attention launch");
+  return RGD_OK;
+}
 template <int D>
 int launch_attn_t(const CUtensorMap& tmK, const CUtensorMap& tmV, const AttnParams& p, const Plan& pl,
                   cudaStream_t st) {
-  static bool done = false;
-  if (int rc = ensure_smem(attn_t_kernel<D>, kSmemLimit, &done)) return rc;
-  attn_t_kernel<D><<<pl.C, kTThreads, pl.smem_bytes, st>>>(tmK, tmV, p);
-  if (cudaError_t e = cudaGetLastError(); e != cudaSuccess) return cuda_error(e, "attention launch");
-  return RGD_OK;
+  switch ((pl.nq + kTQS - 1) / kTQS) {  // softmax sets: one per 8 queries of a job
+    case 1: return launch_attn_t_ns<D, 1>(tmK, tmV, p, pl, st);
+    case 2: return launch_attn_t_ns<D, 2>(tmK, tmV, p, pl, st);
+    case 3: return launch_attn_t_ns<D, 3>(tmK, tmV, p, pl, st);
+    default: return launch_attn_t_ns<D, 4>(tmK, tmV, p, pl, st);
+  }
 }
 
 }  // namespace

@@ -25,11 +25,13 @@
 // operand read from shared memory in MN-major order costs the tensor core
 // twice the cycles of one read from TMEM.
 //
-// Warps: 0-3 and 12-15 softmax (lane quarter w & 3: tokens and, for the V^T
-// copy, head dimensions 32(w & 3)..+31; warps 0-3 take queries 0-15, warps
-// 12-15 queries 16-31), 4-7 piece ends (lane quarter w - 4: head dimensions of
-// O^T; they also write Q), 8 page producer, 9 PV issue of the P residuals,
-// 10 QK issue (and the TMEM allocation), 11 PV issue of the P high parts.
+// Warps: NS = ceil(nq / 8) softmax sets of four warps, set 0 at warps 0-3 and
+// set s > 0 at warps 12 + 4(s - 1) .. +3 (lane quarter w & 3: tokens and, for
+// the V^T copy, head dimensions 32(w & 3)..+31; set s takes queries 8s..8s+7
+// and copies V^T of the group's pages s, s + NS, ...), 4-7 piece ends (lane
+// quarter w - 4: head dimensions of O^T; they also write Q), 8 page producer,
+// 9 PV issue of the P residuals, 10 QK issue (and the TMEM allocation), 11 PV
+// issue of the P high parts.  Query columns past 8 NS are never used.
 // TMEM: S^T x 2 (columns 0-63), O^T of the high parts x 2 by piece (64-127),
 // V^T x 2 (128-255), O^T of the residuals x 2 by piece (256-319); the two O^T
 // accumulate in parallel from two issuing threads and are summed at the piece
@@ -41,7 +43,9 @@ namespace {
 constexpr int kTPages = 8;                  // pages per group: 128 tokens, the MMA's M
 constexpr int kTN = 32;                     // query columns (the MMA's N); jobs with nq <= 32
 constexpr int kTMaxSlots = 6;
-constexpr int kTThreads = 512;
+constexpr int kTQS = 8;                     // queries per softmax set
+template <int NS>
+__host__ __device__ constexpr int t_threads() { return (4 * NS + 8) * 32; }
 constexpr int kTEpi = 4, kTProd = 8, kTPvLo = 9, kTQk = 10, kTPv = 11, kTSoftB = 12;  // first warp of each role
 constexpr int kTTmemCols = 512;
 constexpr int kTSCol = 0;                   // S^T buffers: 2 x 32 columns
@@ -68,8 +72,8 @@ __host__ __device__ inline TLayout t_layout(int nslots, int G, int R) {
   TLayout L;
   L.ring = 0;
   L.q = nslots * t_slot<D>();
-  L.flags = L.q + 2 * t_qbuf<D>();      // [2 sets][2][4] int: a softmax warp needs the maxima moved
-  L.wmax = L.flags + 16 * 4;            // [4][32] per-quarter query maxima of a group
+  L.flags = L.q + 2 * t_qbuf<D>();      // [4 sets][2][4] int: a softmax warp needs the maxima moved
+  L.wmax = L.flags + 32 * 4;            // [4][32] per-quarter query maxima of a group
   L.lw = L.wmax + 4 * kTN * 4;          // [2 pieces][4][32] per-warp query sums
   L.mfin = L.lw + 2 * 4 * kTN * 4;      // [2 pieces][32] query reference maxima at the piece end
   L.mref = L.mfin + 2 * kTN * 4;        // [2 versions][32] current query reference maxima
@@ -129,6 +133,27 @@ __device__ __forceinline__ float transpose_reduce16(float (&v)[16], int lane, Op
   return v[0];
 }
 
+// The same for 8 values per lane: two butterfly steps over the lane quarters,
+// then halving over 8 lanes; lane L ends with the result for index L & 7.
+template <typename Op>
+__device__ __forceinline__ float transpose_reduce8(float (&v)[8], int lane, Op op) {
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] = op(v[i], __shfl_xor_sync(0xffffffffu, v[i], 16));
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] = op(v[i], __shfl_xor_sync(0xffffffffu, v[i], 8));
+#pragma unroll
+  for (int o = 4; o > 0; o >>= 1) {
+    const bool up = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      const float send = up ? v[i] : v[i + o];
+      const float keep = up ? v[i + o] : v[i];
+      v[i] = op(keep, __shfl_xor_sync(0xffffffffu, send, o));
+    }
+  }
+  return v[0];
+}
+
 // P = hi + lo with hi = p truncated to bf16 and lo = (p - hi) truncated to bf16
 // (|p - hi - lo| <= 2^-16 |p|), two values per 32-bit word, the first in the
 // low half.
@@ -139,8 +164,8 @@ __device__ __forceinline__ void split_bf16x2(float p0, float p1, uint32_t& hi, u
   lo = (l0 >> 16) | (l1 & 0xffff0000u);
 }
 
-template <int D>
-__global__ void __launch_bounds__(kTThreads, 1)
+template <int D, int NS>
+__global__ void __launch_bounds__(t_threads<NS>(), 1)
     attn_t_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                   const AttnParams p) {
   constexpr int kTile = kPage * D * 2;  // one K or V page-head tile
@@ -149,6 +174,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
   constexpr int kKArea = t_karea<D>();
   constexpr int kSlot = t_slot<D>();
   constexpr int kQBuf = t_qbuf<D>();
+  constexpr int kThr = t_threads<NS>();
   constexpr uint32_t kIdQK = idesc_bf16_f32(128, kTN, 0, 0);  // A = K, B = Q: both K-major
   constexpr uint32_t kIdPV = idesc_bf16_f32(128, kTN, 0, 1);  // A = V^T from TMEM, B = P^T MN-major
   extern __shared__ uint8_t smem_raw[];
@@ -162,7 +188,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
   __shared__ uint64_t full_bar[kTMaxSlots], empty_bar[kTMaxSlots];
   __shared__ uint64_t s_full[2], s_empty[2], p_full[2], p_empty[2], q_full[2], q_empty[2];
   __shared__ uint64_t o_full[2], o_free[2], ml_full[2], ml_empty[2], mma_done[3];
-  __shared__ int32_t s_abort, s_issued, s_tick, s_wsum[kTThreads / 32];
+  __shared__ int32_t s_abort, s_issued, s_tick, s_wsum[kThr / 32];
   __shared__ uint32_t s_tmem;
   __shared__ PieceIter s_it;
   volatile int32_t* abort_flag = &s_abort;
@@ -180,14 +206,14 @@ __global__ void __launch_bounds__(kTThreads, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&s_empty[i], 8);
-      mbar_init(&p_full[i], 8);
+      mbar_init(&s_empty[i], 4 * NS);
+      mbar_init(&p_full[i], 4 * NS);
       mbar_init(&p_empty[i], 2);
       mbar_init(&q_full[i], 4);
       mbar_init(&q_empty[i], 1);
       mbar_init(&o_full[i], 2);
       mbar_init(&o_free[i], 4);
-      mbar_init(&ml_full[i], 8);
+      mbar_init(&ml_full[i], 4 * NS);
       mbar_init(&ml_empty[i], 4);
       mbar_init(&mma_done[i], 1);
     }
@@ -207,7 +233,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
     const int64_t nb_p = (int64_t)p.G * p.max_pp * 4, nb_s = (int64_t)nrows * p.max_sp * 4;
     const int64_t nb_q = (int64_t)nrows * p.Hq * D * 2;
     const int64_t lp = (nb_p + 127) / 128, ls = (nb_s + 127) / 128, lq = (nb_q + 127) / 128;
-    const int64_t step = (int64_t)p.C * kTThreads;
+    const int64_t step = (int64_t)p.C * kThr;
     for (int64_t l = (int64_t)tid * p.C + c; l < lp + ls + lq; l += step) {
       if (l < lp) prefetch_l2(reinterpret_cast<const uint8_t*>(p.prompt_bt) + l * 128);
       else if (l < lp + ls) prefetch_l2(reinterpret_cast<const uint8_t*>(p.suffix_bt) + (l - lp) * 128);
@@ -215,7 +241,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
     }
   }
   // ---- lengths and activity flags, all loads issued together, kept in shared memory ----
-  for (int r0 = warp * 32; r0 < max(nrows, p.G); r0 += kTThreads) {  // (whole warps: the ballot below)
+  for (int r0 = warp * 32; r0 < max(nrows, p.G); r0 += kThr) {  // (whole warps: the ballot below)
     const int r = r0 + lane;
     int act = 0, sl = 0, pl = 0;
     if (r < nrows) {
@@ -238,7 +264,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
   __syncthreads();
   // a group's pages: its prompt pages if any row of it is active, plus its
   // active rows' suffix pages
-  for (int g = tid; g < p.G; g += kTThreads) {
+  for (int g = tid; g < p.G; g += kThr) {
     int n = 0;
     bool any = false;
     for (int rr = 0; rr < p.rpg; ++rr) {
@@ -253,7 +279,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
   tc_fence_after();
   const uint32_t tmem = s_tmem;
   {  // inclusive prefix sum of gpre[1..G]
-    const int E = (p.G + kTThreads - 1) / kTThreads;
+    const int E = (p.G + kThr - 1) / kThr;
     const int lo = 1 + tid * E, hi = min(p.G + 1, lo + E);
     int sum = 0;
     for (int i = lo; i < hi; ++i) sum += gpre[i];
@@ -267,7 +293,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
     __syncthreads();
     if (tid == 0) {
       int run = 0;
-      for (int w = 0; w < kTThreads / 32; ++w) {
+      for (int w = 0; w < kThr / 32; ++w) {
         const int t = s_wsum[w];
         s_wsum[w] = run;
         run += t;
@@ -463,23 +489,24 @@ __global__ void __launch_bounds__(kTThreads, 1)
     }
   } else if (warp < kTEpi || warp >= kTSoftB) {
     // ============================ softmax ============================
-    // Thread = token t of the group (lane quarter qd); set hb takes queries
-    // 16hb..16hb+15.  The reference maxima of the queries (log2 units) live in
-    // shared memory, two versions per set: a group that moves them writes the
+    // Thread = token t of the group (lane quarter qd); set hs takes queries
+    // 8hs..8hs+7.  The reference maxima of the queries (log2 units) live in
+    // shared memory, two versions: a group that moves a set's maxima writes the
     // other version and the set's threads switch after a barrier, so all use
     // the same reference for a group.  lacc[i] is this thread's running sum of
-    // query 16hb + i.  Before its scores, each thread copies V^T for head
-    // dimension 32qd + lane and the set's 64 tokens of the group into TMEM.
-    const int qd = warp & 3, hb = warp >= kTSoftB ? 1 : 0;
+    // query 8hs + i.  Before its scores, each thread copies V^T for head
+    // dimension 32qd + lane and the set's pages of the group into TMEM.
+    const int qd = warp & 3, hs = warp < 4 ? 0 : 1 + (warp - kTSoftB) / 4;
     const int t = qd * 32 + lane, jp = t >> 4, tip = t & 15;
-    const int q0 = hb * 16;
+    const int q0 = hs * kTQS;
     const uint32_t tl = tmem + ((uint32_t)(qd * 32) << 16);
-    int32_t* flags = reinterpret_cast<int32_t*>(smem + L.flags) + hb * 8;
+    int32_t* flags = reinterpret_cast<int32_t*>(smem + L.flags) + hs * 8;
     float* wmax = reinterpret_cast<float*>(smem + L.wmax);
     float* lw = reinterpret_cast<float*>(smem + L.lw);
     float* mfin = reinterpret_cast<float*>(smem + L.mfin);
     float* mref_s = reinterpret_cast<float*>(smem + L.mref);  // [2 versions][32]
-    auto set_sync = [&]() { asm volatile("bar.sync %0, 128;" ::"r"(hb == 0 ? 1 : 3) : "memory"); };
+    // named barrier of the set's 128 threads (0 is __syncthreads, 2 the piece ends')
+    auto set_sync = [&]() { asm volatile("bar.sync %0, 128;" ::"r"(hs == 0 ? 1 : hs + 2) : "memory"); };
     auto wwait = [&](uint64_t* bar, uint32_t parity) {
       return __all_sync(0xffffffffu, wait_or_abort(bar, parity, abort_flag, p.wait_ns));
     };
@@ -488,10 +515,10 @@ __global__ void __launch_bounds__(kTThreads, 1)
     // V^T copy: this thread's head dimension and its byte within the swizzled V rows
     const int dv = qd * 32 + lane;
     const int vchunk = ((dv & 63) * 2) >> 4;
-    const uint32_t voff = (uint32_t)((dv >> 6) * 2048 + (((dv & 63) * 2) & 15) + hb * 4 * kTile);
-    float lacc[16];
+    const uint32_t voff = (uint32_t)((dv >> 6) * 2048 + (((dv & 63) * 2) & 15));
+    float lacc[kTQS];
 #pragma unroll
-    for (int i = 0; i < 16; ++i) lacc[i] = 0.f;
+    for (int i = 0; i < kTQS; ++i) lacc[i] = 0.f;
     int mv = 0;          // current version of the reference maxima
     bool fresh = true;   // piece start: every reference is -inf (not read from shared memory)
     int gi = 0;
@@ -512,21 +539,25 @@ __global__ void __launch_bounds__(kTThreads, 1)
           if (gi >= 2 && ok && !wwait(&p_empty[sb], (uint32_t)((gi >> 1) - 1) & 1u)) ok = false;
           if (ok && dv < D) {
             const uint32_t vb = sbase + gs * kSlot + kKArea + voff;
-            uint32_t vt[32];
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              // tokens 2i, 2i + 1 of the set's 64: page i / 8, rows (2i) % 16 and + 1
-              const int r = (2 * i) & 15;
-              const uint32_t a0 = vb + (i >> 3) * kTile + r * 128 + (((vchunk ^ r) & 7) << 4);
-              const uint32_t a1 = vb + (i >> 3) * kTile + (r + 1) * 128 + (((vchunk ^ (r + 1)) & 7) << 4);
-              uint16_t x0, x1;
-              asm volatile("ld.shared.u16 %0, [%1];" : "=h"(x0) : "r"(a0));
-              asm volatile("ld.shared.u16 %0, [%1];" : "=h"(x1) : "r"(a1));
-              vt[i] = (uint32_t)x0 | ((uint32_t)x1 << 16);
-            }
             tc_fence_after();
-            tmem_st16(tl + kTVCol + sb * 64 + hb * 32, reinterpret_cast<uint32_t(&)[16]>(vt[0]));
-            tmem_st16(tl + kTVCol + sb * 64 + hb * 32 + 16, reinterpret_cast<uint32_t(&)[16]>(vt[16]));
+#pragma unroll
+            for (int k = 0; k < (kTPages + NS - 1) / NS; ++k) {
+              const int jj = hs + k * NS;  // a page of the group: tokens 16jj..16jj+15
+              if (jj < kTPages) {
+                uint32_t vt[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                  const int r = 2 * i;
+                  const uint32_t a0 = vb + jj * kTile + r * 128 + (((vchunk ^ r) & 7) << 4);
+                  const uint32_t a1 = vb + jj * kTile + (r + 1) * 128 + (((vchunk ^ (r + 1)) & 7) << 4);
+                  uint16_t x0, x1;
+                  asm volatile("ld.shared.u16 %0, [%1];" : "=h"(x0) : "r"(a0));
+                  asm volatile("ld.shared.u16 %0, [%1];" : "=h"(x1) : "r"(a1));
+                  vt[i] = (uint32_t)x0 | ((uint32_t)x1 << 16);
+                }
+                tmem_st8(tl + kTVCol + sb * 64 + jj * 8, vt);
+              }
+            }
           }
           int tok = 0, sel = -1;
           if (ok && has) {
@@ -536,9 +567,9 @@ __global__ void __launch_bounds__(kTThreads, 1)
           }
           if (ok && !wwait(&s_full[sb], (uint32_t)(gi >> 1) & 1u)) ok = false;
           tc_fence_after();
-          float sc[16];
+          float sc[kTQS];
           if (ok) {
-            tmem_ld16(tl + kTSCol + sb * kTN + q0, reinterpret_cast<uint32_t(&)[16]>(sc));
+            tmem_ld8(tl + kTSCol + sb * kTN + q0, reinterpret_cast<uint32_t(&)[kTQS]>(sc));
             tmem_ld_wait();
           }
           tc_fence_before();
@@ -552,7 +583,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
           const float* mr = mref_s + mv * kTN + q0;
           bool ex = false;
 #pragma unroll
-          for (int q = 0; q < 16; q += 4) {
+          for (int q = 0; q < kTQS; q += 4) {
             const float4 m4 = fresh ? make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY)
                                     : *reinterpret_cast<const float4*>(mr + q);
             const float mm[4] = {m4.x, m4.y, m4.z, m4.w};
@@ -570,20 +601,20 @@ __global__ void __launch_bounds__(kTThreads, 1)
           if ((fl[0] | fl[1] | fl[2] | fl[3]) != 0) {
             // this warp's query maxima (lane i: query q0 + i), then the new
             // reference of each query from the four warps and its factor f
-            float v[16];
+            float v[kTQS];
 #pragma unroll
-            for (int q = 0; q < 16; ++q) v[q] = sc[q];
-            const float wm = transpose_reduce16(v, lane, [](float x, float y) { return fmaxf(x, y); });
-            if (lane < 16) wmax[qd * kTN + q0 + lane] = wm;
+            for (int q = 0; q < kTQS; ++q) v[q] = sc[q];
+            const float wm = transpose_reduce8(v, lane, [](float x, float y) { return fmaxf(x, y); });
+            if (lane < kTQS) wmax[qd * kTN + q0 + lane] = wm;
             set_sync();
-            const int qi = q0 + (lane & 15);
-            const float mo = fresh ? -INFINITY : mr[lane & 15];
+            const int qi = q0 + (lane & (kTQS - 1));
+            const float mo = fresh ? -INFINITY : mr[lane & (kTQS - 1)];
             const float mn = fmaxf(fmaxf(mo, wmax[qi]), fmaxf(fmaxf(wmax[kTN + qi], wmax[2 * kTN + qi]),
                                                              wmax[3 * kTN + qi]));
             const float fq = mo == -INFINITY ? 0.f : exp2f(mo - mn);
-            if (qd == 0 && lane < 16) mref_s[(mv ^ 1) * kTN + qi] = mn;
+            if (qd == 0 && lane < kTQS) mref_s[(mv ^ 1) * kTN + qi] = mn;
 #pragma unroll
-            for (int q = 0; q < 16; ++q) lacc[q] *= __shfl_sync(0xffffffffu, fq, q);
+            for (int q = 0; q < kTQS; ++q) lacc[q] *= __shfl_sync(0xffffffffu, fq, q);
             // O^T already holds this piece's earlier groups: once their PV is
             // done, the set's query columns (this warp's 32 head dimensions) are scaled
             if (k0 > 0) {
@@ -594,13 +625,13 @@ __global__ void __launch_bounds__(kTThreads, 1)
 #pragma unroll
                 for (int part = 0; part < 2; ++part) {
                   const uint32_t oc = tl + (part ? kTOLoCol : kTOCol) + ob * kTN + q0;
-                  uint32_t o16[16];
-                  tmem_ld16(oc, o16);
+                  uint32_t o8[kTQS];
+                  tmem_ld8(oc, o8);
                   tmem_ld_wait();
 #pragma unroll
-                  for (int u = 0; u < 16; ++u)
-                    o16[u] = __float_as_uint(__uint_as_float(o16[u]) * __shfl_sync(0xffffffffu, fq, u));
-                  tmem_st16(oc, o16);
+                  for (int u = 0; u < kTQS; ++u)
+                    o8[u] = __float_as_uint(__uint_as_float(o8[u]) * __shfl_sync(0xffffffffu, fq, u));
+                  tmem_st8(oc, o8);
                 }
               }
             }
@@ -609,10 +640,10 @@ __global__ void __launch_bounds__(kTThreads, 1)
             fresh = false;
           }
           // P = 2^(s - m) in bf16 high part + residual (ex2 of -inf is +0)
-          uint32_t ph[8], plo[8];
+          uint32_t ph[kTQS / 2], plo[kTQS / 2];
           const float* mc = mref_s + mv * kTN + q0;
 #pragma unroll
-          for (int q = 0; q < 16; q += 4) {
+          for (int q = 0; q < kTQS; q += 4) {
             const float4 m4 = fresh ? make_float4(0.f, 0.f, 0.f, 0.f) : *reinterpret_cast<const float4*>(mc + q);
             const float mm[4] = {m4.x, m4.y, m4.z, m4.w};
 #pragma unroll
@@ -625,16 +656,11 @@ __global__ void __launch_bounds__(kTThreads, 1)
               split_bf16x2(p0, p1, ph[(q + u) / 2], plo[(q + u) / 2]);
             }
           }
-          // the group's slot is the P^T area once its QK is done (this set's 32 bytes of each row)
+          // the group's slot is the P^T area once its QK is done (this set's 16 bytes of each row)
           if (ok) {
             const uint32_t pbase = sbase + gs * kSlot;
-#pragma unroll
-            for (int ch = 0; ch < 2; ++ch) {
-              st_shared_v4(pbase + sw64_off(t, 2 * hb + ch), ph[4 * ch], ph[4 * ch + 1], ph[4 * ch + 2],
-                           ph[4 * ch + 3]);
-              st_shared_v4(pbase + kTPHalf + sw64_off(t, 2 * hb + ch), plo[4 * ch], plo[4 * ch + 1],
-                           plo[4 * ch + 2], plo[4 * ch + 3]);
-            }
+            st_shared_v4(pbase + sw64_off(t, hs), ph[0], ph[1], ph[2], ph[3]);
+            st_shared_v4(pbase + kTPHalf + sw64_off(t, hs), plo[0], plo[1], plo[2], plo[3]);
           }
           tmem_st_wait();            // V^T (and any O rescale) are in TMEM
           fence_proxy_async_smem();  // the MMAs read P^T through the async proxy
@@ -645,15 +671,15 @@ __global__ void __launch_bounds__(kTThreads, 1)
         }
         // piece end: per-warp query sums and the reference maxima to the epilogue warps
         if (pc >= 2 && ok && !wwait(&ml_empty[ob], (uint32_t)((pc >> 1) - 1) & 1u)) ok = false;
-        const float ls = transpose_reduce16(lacc, lane, [](float x, float y) { return x + y; });
-        if (lane < 16) {
+        const float ls = transpose_reduce8(lacc, lane, [](float x, float y) { return x + y; });
+        if (lane < kTQS) {
           lw[(ob * 4 + qd) * kTN + q0 + lane] = ls;
           if (qd == 0) mfin[ob * kTN + q0 + lane] = fresh ? -INFINITY : mref_s[mv * kTN + q0 + lane];
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&ml_full[ob]);
 #pragma unroll
-        for (int q = 0; q < 16; ++q) lacc[q] = 0.f;
+        for (int q = 0; q < kTQS; ++q) lacc[q] = 0.f;
         fresh = true;
         ++pc;
       }

@@ -94,6 +94,19 @@ def test_query_copy_counts(gpu_lib, D, rpg, Hq, Hkv, ctas):
     _check(case, _run(case, num_ctas=ctas))
 
 
+@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("rpg", [1, 3, 5, 7, 8])
+@pytest.mark.parametrize("ctas", [0, 7])
+def test_softmax_set_counts(gpu_lib, D, rpg, ctas):
+    # queries per kv head 4, 12, 20, 28 and 32: one to four sets of eight query
+    # columns in the transposed kernel (the last set partly or wholly padding
+    # for 4, 12, 20 and 28), jobs whole in one block and split over blocks
+    G = 3
+    slens = [(11 * i) % 90 for i in range(G * rpg)]
+    case = workloads.make_attn_case("sets", G, rpg, 32, 8, D, [0, 45, 230], slens, seed=100 + rpg + D)
+    _check(case, _run(case, num_ctas=ctas))
+
+
 def test_masked_rows_and_groups(gpu_lib):
     active = np.array([1, 0, 1, 0, 0, 0, 0, 1, 1], np.uint8)  # group 1 fully masked
     case = workloads.make_attn_case("mask", 3, 3, 8, 2, 128, [50, 70, 90], [3, 4, 5, 6, 7, 8, 0, 0, 20],
