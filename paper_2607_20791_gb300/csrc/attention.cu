@@ -190,6 +190,13 @@ struct Job {
 };
 
 // The job containing global page x (x < total pages).
+// a / b for a >= 0, b > 0: 32-bit division when both fit (the usual case;
+// 64-bit division is a long instruction sequence on the GPU).
+__device__ __forceinline__ int64_t div_nn(int64_t a, int64_t b) {
+  if (((uint64_t)a | (uint64_t)b) >> 32 == 0) return (int64_t)((uint32_t)a / (uint32_t)b);
+  return a / b;
+}
+
 __device__ Job job_at(const AttnParams& p, const int32_t* gpre, int64_t x) {
   int lo = 0, hi = p.G - 1;  // largest g with Hkv * gpre[g] <= x
   while (lo < hi) {
@@ -201,7 +208,7 @@ __device__ Job job_at(const AttnParams& p, const int32_t* gpre, int64_t x) {
   j.g = lo;
   j.n = gpre[lo + 1] - gpre[lo];
   const int64_t base = (int64_t)p.Hkv * gpre[lo];
-  j.h = (int)((x - base) / j.n);
+  j.h = (int)div_nn(x - base, j.n);
   j.start = base + (int64_t)j.h * j.n;
   return j;
 }
@@ -220,7 +227,7 @@ __device__ Job next_job(const AttnParams& p, const int32_t* gpre, Job j) {
 }
 
 // Block whose page range contains global page x (ranges [floor(cT/C), floor((c+1)T/C))).
-__device__ __forceinline__ int cta_of(int64_t x, int64_t T, int C) { return (int)(((x + 1) * C - 1) / T); }
+__device__ __forceinline__ int cta_of(int64_t x, int64_t T, int C) { return (int)div_nn((x + 1) * C - 1, T); }
 
 // A block's job pieces in the order it works on them: the job at the start of
 // its range, then the job at the end, then the whole jobs in between.  Only the
@@ -390,6 +397,10 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
     tmem_alloc(&s_tmem, kTmemCols);
     tmem_relinquish();
   }
+  if (warp == kProducerWarp && lane == 0) {  // the copies' descriptors, fetched while the set-up runs
+    prefetch_tensormap(&tmK);
+    prefetch_tensormap(&tmV);
+  }
   // ---- page counts per group and their exclusive prefix sum (every block) ----
   // The lengths and activity flags are read once, all loads issued together
   // (one global-memory latency), and kept in shared memory for the producer.
@@ -464,8 +475,8 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
   // pages are divided over Ceff = min(C, T) blocks so that every working block
   // has at least one page (a job's pieces are then exactly the blocks first..last)
   const int Ceff = (int)min((int64_t)p.C, T);
-  const int64_t b = c < Ceff ? (int64_t)c * T / Ceff : T;
-  const int64_t e = c < Ceff ? (int64_t)(c + 1) * T / Ceff : T;
+  const int64_t b = c < Ceff ? div_nn((int64_t)c * T, Ceff) : T;
+  const int64_t e = c < Ceff ? div_nn((int64_t)(c + 1) * T, Ceff) : T;
   // the piece order, kept in shared memory (read at piece boundaries only)
   __shared__ PieceIter s_it;
   if (tid == 0 && b < e) s_it = piece_iter(p, gpre, b, e);
@@ -488,10 +499,6 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
     // pages of earlier rounds, so neither warp can hold up the other.
     const int pw = warp - kProducerWarp;
     if (b < e) {
-      if (lane == 0 && pw == 0) {
-        prefetch_tensormap(&tmK);
-        prefetch_tensormap(&tmV);
-      }
       const uint64_t pol = policy_evict_first();
       const PieceIter& it = s_it;
       int gbase = 0;  // groups started before sequence position ib

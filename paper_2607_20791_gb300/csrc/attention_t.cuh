@@ -226,6 +226,10 @@ __global__ void __launch_bounds__(t_threads<NS>(), 1)
     tmem_alloc(&s_tmem, kTTmemCols);
     tmem_relinquish();
   }
+  if (warp == kTProd && lane == 0) {  // the copies' descriptors, fetched while the set-up runs
+    prefetch_tensormap(&tmK);
+    prefetch_tensormap(&tmV);
+  }
   // This block's share of the block tables and queries is asked of L2 while the
   // lengths load (each line once over the grid), so that the first block-table
   // and query loads of every block find them there.
@@ -278,7 +282,17 @@ __global__ void __launch_bounds__(t_threads<NS>(), 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = s_tmem;
-  {  // inclusive prefix sum of gpre[1..G]
+  if (p.G <= 32) {  // inclusive prefix sum of gpre[1..G]: one warp (uniform branch)
+    if (warp == 0) {
+      int incl = lane < p.G ? gpre[lane + 1] : 0;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += v;
+      }
+      if (lane < p.G) gpre[lane + 1] = incl;
+    }
+  } else {  // the same over every thread
     const int E = (p.G + kThr - 1) / kThr;
     const int lo = 1 + tid * E, hi = min(p.G + 1, lo + E);
     int sum = 0;
@@ -309,8 +323,8 @@ __global__ void __launch_bounds__(t_threads<NS>(), 1)
   __syncthreads();
   const int64_t T = (int64_t)p.Hkv * gpre[p.G];
   const int Ceff = (int)min((int64_t)p.C, T);
-  const int64_t b = c < Ceff ? (int64_t)c * T / Ceff : T;
-  const int64_t e = c < Ceff ? (int64_t)(c + 1) * T / Ceff : T;
+  const int64_t b = c < Ceff ? div_nn((int64_t)c * T, Ceff) : T;
+  const int64_t e = c < Ceff ? div_nn((int64_t)(c + 1) * T, Ceff) : T;
   if (tid == 0 && b < e) s_it = piece_iter(p, gpre, b, e);
   __syncthreads();
 
@@ -323,10 +337,6 @@ __global__ void __launch_bounds__(t_threads<NS>(), 1)
     // before the previous round's copies wait for their slots, so the
     // block-table loads are in flight while the warp waits.
     if (b < e) {
-      if (lane == 0) {
-        prefetch_tensormap(&tmK);
-        prefetch_tensormap(&tmV);
-      }
       const uint64_t pol = policy_evict_first();
       const PieceIter& it = s_it;
       struct Pg {
