@@ -53,7 +53,7 @@ def _run_loop(P, eos, groups, vocab, steps, c, k, rho, max_len, seed, dtype="f32
     mass = torch.empty(groups, dtype=torch.float32, device="cuda")
     ref = [ogate.GateState() for _ in range(groups)]
     ref_active = np.ones(groups * rpg, np.uint8)
-    boundary = soft = 0
+    boundary = soft = deep = 0
     for step in range(steps):
         l32 = (rng.standard_normal((groups, vocab)) * scale).astype(np.float32)
         l32 = np.round(l32, 1)  # ties
@@ -79,6 +79,9 @@ def _run_loop(P, eos, groups, vocab, steps, c, k, rho, max_len, seed, dtype="f32
                 continue
             if r.soft:
                 soft += 1
+                # more than the four candidates the kernel's one pass ranks are
+                # inside the top K: the kernel sorts them and searches the rest
+                deep += len(r.a_ref) > 4
                 assert abs(m_gpu[g] - r.mass) <= 1e-5 * r.mass + 1e-7, (step, g, m_gpu[g], r.mass)
             else:
                 assert m_gpu[g] == -1.0
@@ -87,7 +90,7 @@ def _run_loop(P, eos, groups, vocab, steps, c, k, rho, max_len, seed, dtype="f32
                 # only a continue/discard flip at the rho boundary is allowed
                 assert r.soft and abs(r.mass - rho) <= 2e-5 * max(rho, r.mass), (step, g, t_gpu[g], exp_tok)
                 boundary += 1
-                return boundary, soft  # the two runs have diverged; stop comparing this loop
+                return boundary, soft, deep  # the two runs have diverged; stop comparing this loop
             assert got["decision"][g] == ref[g].decision, (step, g)
             assert got["done"][g] == int(ref[g].done), (step, g)
             assert got["decisive_step"][g] == ref[g].decisive_step, (step, g)
@@ -95,29 +98,40 @@ def _run_loop(P, eos, groups, vocab, steps, c, k, rho, max_len, seed, dtype="f32
         ref_active = ogate.row_mask_update(ref, rpg, ref_active)
         assert np.array_equal(active.cpu().numpy(), ref_active), step
     trie.close()
-    return boundary, soft
+    return boundary, soft, deep
 
 
 @pytest.mark.parametrize("seed", range(4))
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 def test_soft_gate_loops_small_vocab(gpu_lib, seed, dtype):
     P = workloads.make_refusal_set(12, 2, 6, 300, seed, avoid=[7])
-    boundary, soft = _run_loop(P, eos=7, groups=24, vocab=300, steps=8, c=5, k=20, rho=0.05, max_len=12,
+    boundary, soft, deep = _run_loop(P, eos=7, groups=24, vocab=300, steps=8, c=5, k=20, rho=0.05, max_len=12,
                                seed=seed, dtype=dtype)
+    assert soft > 0 and boundary <= 1
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_soft_gate_unaligned_rows(gpu_lib, dtype):
+    # vocabulary 301: row starts off 16-byte boundaries, so the kernel reads
+    # single elements instead of staging 16-byte vectors
+    P = workloads.make_refusal_set(12, 2, 6, 301, 3, avoid=[7])
+    boundary, soft, deep = _run_loop(P, eos=7, groups=24, vocab=301, steps=8, c=5, k=20, rho=0.05, max_len=12,
+                                     seed=3, dtype=dtype)
     assert soft > 0 and boundary <= 1
 
 
 def test_soft_gate_many_candidates_and_large_k(gpu_lib):
     # 600 refusal sequences: the root has hundreds of children; K = 100 needs several ranking passes
     P = workloads.make_refusal_set(600, 2, 8, 4000, 5)
-    boundary, soft = _run_loop(P, eos=-1, groups=16, vocab=4000, steps=5, c=3, k=100, rho=0.02, max_len=8,
-                               seed=5, boost=0.9, scale=1.0)
+    boundary, soft, deep = _run_loop(P, eos=-1, groups=16, vocab=4000, steps=5, c=3, k=100, rho=0.02, max_len=8,
+                                     seed=5, boost=0.9, scale=1.0)
     assert soft > 0 and boundary <= 1
+    assert deep > 0  # the sort-and-search path ran
 
 
 def test_soft_gate_llama_vocab(gpu_lib):
     P = workloads.make_refusal_set(64, 2, 8, 128256, 9, avoid=[128009])
-    boundary, soft = _run_loop(P, eos=128009, groups=16, vocab=128256, steps=4, c=4, k=40, rho=0.1, max_len=32,
+    boundary, soft, deep = _run_loop(P, eos=128009, groups=16, vocab=128256, steps=4, c=4, k=40, rho=0.1, max_len=32,
                                seed=9, boost=0.8)
     assert soft > 0 and boundary <= 1
 
