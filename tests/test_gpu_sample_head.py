@@ -66,6 +66,16 @@ def test_sweep_small_batches(gpu_lib, batch, vocab, dtype):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("batch", [128, 300, 500])
+def test_several_waves(gpu_lib, batch, dtype):
+    # 128, 300 and 500 rows at 8 CTAs per row are more CTAs than the device
+    # holds at once (5 per SM): clusters run in several waves; every row and
+    # kept mask compared
+    case = workloads.head_sweep(batch, 32000, dtype, seed=7 + batch)
+    assert _check(case, _run(case)) == 0
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("vocab", [1, 7, 33, 1000, 4097, 32001])
 def test_ragged_vocab(gpu_lib, vocab, dtype):
     # rows start at unaligned addresses; slices end in ragged tails; tiny vocabularies
