@@ -321,6 +321,73 @@ __device__ __forceinline__ bool wait_slot_gen(int32_t* gen, int32_t want, volati
   }
 }
 
+// The merge of a split job whose other pieces' partials do not fit the
+// prefetch area: every piece's partial read straight from global memory (L2,
+// past L1) after the job's count is complete; each of the n_et epilogue
+// threads folds its kU float4 columns of O over the pieces in order (the loads
+// of one piece for all of them in flight at once) and writes the output.  Out
+// of line, so that its registers do not crowd the kernel's other code.
+template <int D>
+__device__ __noinline__ void merge_from_l2(const float2* slot_ml, const float* slot_o, __nv_bfloat16* out, float* lse,
+                                           int nq, int gq, int rpg, int Hq, int g, int h, int jj, int first,
+                                           int last, int et, int n_et, const uint32_t* rowbits, bool good) {
+  constexpr int kU = 4;  // columns per thread per pass
+  const int mls = ml_stride(nq), n4 = nq * (D / 4);
+  for (int b0 = 0; b0 < n4; b0 += kU * n_et) {
+    const int base = b0 + et;
+    float Mm[kU], Lm[kU];
+    float4 acc[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      Mm[u] = -INFINITY;
+      Lm[u] = 0.f;
+      acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    for (int s2 = first; s2 <= last && good; ++s2) {
+      const int64_t sl = (int64_t)s2 + jj;
+      float2 ml[kU];
+      float4 v[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int it = base + u * n_et;
+        ml[u] = make_float2(-INFINITY, 0.f);
+        v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (it < n4) {
+          const int i = it / (D / 4), c4 = it % (D / 4);
+          ml[u] = __ldcg(slot_ml + sl * mls + i);
+          v[u] = __ldcg(reinterpret_cast<const float4*>(slot_o + (sl * nq + i) * D) + c4);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        if (ml[u].y == 0.f) continue;
+        const float Mn = fmaxf(Mm[u], ml[u].x);
+        const float f = Mm[u] == -INFINITY ? 0.f : exp2f(Mm[u] - Mn), w = exp2f(ml[u].x - Mn);
+        Lm[u] = Lm[u] * f + w * ml[u].y;
+        acc[u].x = acc[u].x * f + w * v[u].x;
+        acc[u].y = acc[u].y * f + w * v[u].y;
+        acc[u].z = acc[u].z * f + w * v[u].z;
+        acc[u].w = acc[u].w * f + w * v[u].w;
+        Mm[u] = Mn;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int it = base + u * n_et;
+      if (!good || it >= n4) break;  // (after an abort the outputs are not written)
+      const int i = it / (D / 4), c4 = it % (D / 4);
+      const int rr2 = g * rpg + i / gq, hq2 = h * gq + i % gq;
+      if (!((rowbits[rr2 >> 5] >> (rr2 & 31)) & 1u)) continue;
+      const float iv = Lm[u] > 0.f ? 1.f / Lm[u] : 0.f;
+      uint2 pk2;
+      pk2.x = pack_bf16x2(acc[u].x * iv, acc[u].y * iv);
+      pk2.y = pack_bf16x2(acc[u].z * iv, acc[u].w * iv);
+      reinterpret_cast<uint2*>(out + ((int64_t)rr2 * Hq + hq2) * D)[c4] = pk2;
+      if (lse && c4 == 0) lse[(int64_t)rr2 * Hq + hq2] = Lm[u] > 0.f ? (Mm[u] + log2f(Lm[u])) * kLn2 : -INFINITY;
+    }
+  }
+}
+
 template <int D, int R>
 __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
@@ -915,71 +982,9 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
     // each thread folds it into its items (item = 4 output columns of one
     // query), kU items at a time: with piece s holding the unnormalised o_s and
     // (m_s, l_s) in log2 units, out = sum 2^(m_s - M) o_s / sum 2^(m_s - M) l_s.
-    auto merge_staged = [&](const Job& jb, int jj, int first, int last, int et, int n_et, bool copier) {
-      constexpr int kU = R == 4 ? 8 : 2;  // (more fit in the registers of the 4-copy layout only)
-      const int mls = ml_stride(nq), n4 = nq * (D / 4);
-      bool good = true;  // no wait has given up (the barriers below are passed regardless)
-      for (int b0 = 0; b0 < n4; b0 += kU * n_et) {  // (the same trip counts in every thread)
-        const int base = b0 + et;
-        float Mm[kU], Lm[kU];
-        float4 acc[kU];
-#pragma unroll
-        for (int u = 0; u < kU; ++u) {
-          Mm[u] = -INFINITY;
-          Lm[u] = 0.f;
-          acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-        for (int s2 = first; s2 <= last; ++s2) {
-          const int64_t sl = (int64_t)s2 + jj;
-          if (copier && __all_sync(0xffffffffu, good && !*abort_flag)) {
-            if (lane == 0) {
-              mbar_arrive_expect_tx(&pref_bar, (uint32_t)(nq * D * 4 + mls * 8));
-              ++s_pref_n;
-            }
-            __syncwarp();
-            fence_proxy_async_global();
-            for (int i = lane; i <= nq; i += 32) {
-              if (i < nq) bulk_load(pref_o + i * (D + 4), p.slot_o + (sl * nq + i) * D, D * 4, &pref_bar);
-              else bulk_load(pref_ml, p.slot_ml + sl * mls, mls * 8, &pref_bar);
-            }
-          }
-          good = wwait(&pref_bar, (uint32_t)n_pref & 1u, abort_flag) && good;  // (after an abort: at once)
-          ++n_pref;
-#pragma unroll
-          for (int u = 0; u < kU; ++u) {
-            const int it = base + u * n_et;
-            if (!good || it >= n4) break;
-            const int i = it / (D / 4), c4 = it % (D / 4);
-            const float2 ml = pref_ml[i];
-            if (ml.y == 0.f) continue;
-            const float4 v = reinterpret_cast<const float4*>(pref_o + i * (D + 4))[c4];
-            const float Mn = fmaxf(Mm[u], ml.x);
-            const float f = Mm[u] == -INFINITY ? 0.f : exp2f(Mm[u] - Mn), w = exp2f(ml.x - Mn);
-            Lm[u] = Lm[u] * f + w * ml.y;
-            acc[u].x = acc[u].x * f + w * v.x;
-            acc[u].y = acc[u].y * f + w * v.y;
-            acc[u].z = acc[u].z * f + w * v.z;
-            acc[u].w = acc[u].w * f + w * v.w;
-            Mm[u] = Mn;
-          }
-          epi_sync();  // the area is read before the next piece's copies
-        }
-#pragma unroll
-        for (int u = 0; u < kU; ++u) {
-          const int it = base + u * n_et;
-          if (!good || it >= n4) break;  // (after an abort the outputs are not written)
-          const int i = it / (D / 4), c4 = it % (D / 4);
-          const int rr2 = jb.g * p.rpg + i / gq, hq2 = jb.h * gq + i % gq;
-          if (!((rowbits[rr2 >> 5] >> (rr2 & 31)) & 1u)) continue;
-          const float iv = Lm[u] > 0.f ? 1.f / Lm[u] : 0.f;
-          uint2 pk2;
-          pk2.x = pack_bf16x2(acc[u].x * iv, acc[u].y * iv);
-          pk2.y = pack_bf16x2(acc[u].z * iv, acc[u].w * iv);
-          reinterpret_cast<uint2*>(p.out + ((int64_t)rr2 * p.Hq + hq2) * D)[c4] = pk2;
-          if (p.lse && c4 == 0)
-            p.lse[(int64_t)rr2 * p.Hq + hq2] = Lm[u] > 0.f ? (Mm[u] + log2f(Lm[u])) * kLn2 : -INFINITY;
-        }
-      }
+    auto merge_staged = [&](const Job& jb, int jj, int first, int last, int et, int n_et) {
+      merge_from_l2<D>(p.slot_ml, p.slot_o, p.out, p.lse, nq, gq, p.rpg, p.Hq, jb.g, jb.h, jj, first, last, et, n_et,
+                       rowbits, !*abort_flag);
     };
     // the next piece's Q, then this piece's end (epilogue warps)
     auto run_epilogue = [&](const Job& cur, int pc, bool more, const Job& nxt) {
@@ -1305,7 +1310,7 @@ __global__ void __launch_bounds__(Roles<R>::kThreads, 1)
       epi_sync();
       if (s_last == 1) {
         __threadfence();
-        merge_staged(cur, j, first, last, et, n_et, watcher);
+        merge_staged(cur, j, first, last, et, n_et);
       }
       if (et == 0) p.ticket[j] = 0;
       epi_sync();  // (the prefetch area and s_last are reused at the next piece)
